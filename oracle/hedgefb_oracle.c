@@ -1,0 +1,382 @@
+/*
+ * hedgefb_oracle.c -- plain, slow, fp64 CPU restatement of the HedgeSpec
+ * panoramic-feedback path ("Not-a-Bandit", arXiv 2510.20064).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the oracle that the CUDA library is
+ * checked against.  Only the test-suite, the smoke check and the CPU-baseline
+ * leg of the benchmark may load it.  It shares no code, header, table or
+ * constant with the CUDA library and never calls into it.
+ *
+ * Every function evaluates the paper's definition directly, in fp64, with
+ * plain loops in index order:
+ *   - Thm 1 (Sec. 2.2):      alpha = sum_x min(p(x), q(x)) = 1 - TV(p, q)
+ *   - Thm 2 with L = 1 and a greedy target (Sec. 2.3): greedy alpha is the
+ *                            indicator that the two argmaxes agree
+ *   - Thm 3 (Sec. 3.2):      counterfactual acceptance-length estimator
+ *   - Sec. 3.3 / App. B.3:   length loss and acceptance-rate loss
+ *   - App. B.1 remark:       Hedge, w_i <- w_i exp(-eta l_i), normalised
+ *   - App. D.6 (Fig. "NormalHedge"): NormalHedge regret update, scale c and
+ *                            weights
+ * Input logits are read as the very bytes the GPU reads: bf16 is widened by
+ * a 16-bit shift, fp16 by its IEEE-754 binary16 definition, fp32 as is; all
+ * three conversions to double are exact.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+enum { ORC_BF16 = 0, ORC_FP16 = 1, ORC_FP32 = 2 };
+enum { ORC_OK = 0, ORC_BADARG = 1, ORC_NONFINITE = 4 };
+enum { ORC_LOSS_LENGTH = 0, ORC_LOSS_ACCEPT = 1 };
+enum { ORC_HEDGE = 0, ORC_NORMALHEDGE = 1 };
+
+/* ---- exact decode of one stored logit -------------------------------- */
+
+static double decode_bf16(uint16_t h) {
+  uint32_t bits = ((uint32_t)h) << 16;  /* bf16 is the top half of binary32 */
+  float f;
+  memcpy(&f, &bits, sizeof f);
+  return (double)f;
+}
+
+static double decode_fp16(uint16_t h) {
+  int sign = (h >> 15) & 1;
+  int expo = (h >> 10) & 0x1f;
+  int mant = h & 0x3ff;
+  double v;
+  if (expo == 0)
+    v = ldexp((double)mant, -24);                  /* subnormal: mant * 2^-24 */
+  else if (expo == 31)
+    v = mant ? NAN : INFINITY;
+  else
+    v = ldexp((double)(mant + 1024), expo - 25);   /* (1 + mant/1024) 2^(e-15) */
+  return sign ? -v : v;
+}
+
+double orc_decode(const void* base, int dtype, int64_t idx) {
+  if (dtype == ORC_BF16) return decode_bf16(((const uint16_t*)base)[idx]);
+  if (dtype == ORC_FP16) return decode_fp16(((const uint16_t*)base)[idx]);
+  return (double)((const float*)base)[idx];
+}
+
+/* ---- one row: softmax at temperature T (the p(.) / q(.) of Thm 1) ---- */
+
+/* A row is usable when it holds no NaN, no +inf and at least one finite
+ * value; -inf entries are masked vocabulary and have probability 0. */
+static int row_ok(const void* row, int dtype, int V) {
+  int any_finite = 0;
+  for (int v = 0; v < V; ++v) {
+    double z = orc_decode(row, dtype, v);
+    if (isnan(z) || z == INFINITY) return 0;
+    if (z != -INFINITY) any_finite = 1;
+  }
+  return any_finite;
+}
+
+/* P[v] = exp(z_v/T - lse),  lse = m + log sum_v exp(z_v/T - m),  m = max z/T. */
+int orc_row_probs(const void* row, int dtype, int V, double T, double* P) {
+  if (!row_ok(row, dtype, V)) {
+    for (int v = 0; v < V; ++v) P[v] = NAN;
+    return ORC_NONFINITE;
+  }
+  double m = -INFINITY;
+  for (int v = 0; v < V; ++v) {
+    double s = orc_decode(row, dtype, v) / T;
+    if (s > m) m = s;
+  }
+  double sum = 0.0;
+  for (int v = 0; v < V; ++v) sum += exp(orc_decode(row, dtype, v) / T - m);
+  double lse = m + log(sum);
+  for (int v = 0; v < V; ++v) P[v] = exp(orc_decode(row, dtype, v) / T - lse);
+  return ORC_OK;
+}
+
+/* First index of the largest stored logit (ties -> lowest index; -0 == +0).
+ * Returns -1 for an unusable row. */
+int orc_row_argmax(const void* row, int dtype, int V) {
+  if (!row_ok(row, dtype, V)) return -1;
+  int best = 0;
+  double bz = orc_decode(row, dtype, 0);
+  for (int v = 1; v < V; ++v) {
+    double z = orc_decode(row, dtype, v);
+    if (z > bz) { bz = z; best = v; }
+  }
+  return best;
+}
+
+/* Thm 1: acceptance probability of one draft position = sum_x min(p, q). */
+double orc_overlap(const double* P, const double* Q, int V) {
+  double a = 0.0;
+  for (int v = 0; v < V; ++v) a += (P[v] < Q[v]) ? P[v] : Q[v];
+  return a;
+}
+
+/* Thm 1, right-hand side: TV(p, q) = 1/2 sum_x |p(x) - q(x)|. */
+double orc_tv(const double* P, const double* Q, int V) {
+  double t = 0.0;
+  for (int v = 0; v < V; ++v) t += fabs(P[v] - Q[v]);
+  return 0.5 * t;
+}
+
+/* alpha for one (target row, drafter row) pair.
+ * Stochastic: Thm 1.  Greedy: Thm 2 with branching L = 1 under a greedy
+ * (argmax) target -- the drafted token is accepted iff both argmaxes agree. */
+int orc_alpha_pair(const void* zt, const void* zd, int dtype, int V, double T,
+                   int greedy, double* alpha) {
+  if (greedy) {
+    int jt = orc_row_argmax(zt, dtype, V), jd = orc_row_argmax(zd, dtype, V);
+    if (jt < 0 || jd < 0) { *alpha = NAN; return ORC_NONFINITE; }
+    *alpha = (jt == jd) ? 1.0 : 0.0;
+    return ORC_OK;
+  }
+  double* P = (double*)malloc(sizeof(double) * (size_t)V);
+  double* Q = (double*)malloc(sizeof(double) * (size_t)V);
+  int st = orc_row_probs(zt, dtype, V, T, P);
+  st |= orc_row_probs(zd, dtype, V, T, Q);
+  *alpha = st ? NAN : orc_overlap(P, Q, V);
+  free(P);
+  free(Q);
+  return st ? ORC_NONFINITE : ORC_OK;
+}
+
+/* ---- Thm 3: counterfactual acceptance length ------------------------- */
+
+/* Sum of prefix products: 1 + sum_{k=1..K} prod_{j<=k} gamma_j.
+ * gamma[0..K-1] are gamma_1..gamma_K; gamma_{K+1} := 0 is implicit. */
+double orc_elen_prefix(const double* gamma, int K) {
+  double e = 1.0, prod = 1.0;
+  for (int k = 0; k < K; ++k) {
+    prod *= gamma[k];
+    e += prod;
+  }
+  return e;
+}
+
+/* The estimator exactly as Thm 3 prints it:
+ * sum_{k=1..K+1} k (1 - gamma_k) prod_{j=1..k-1} gamma_j,  gamma_{K+1} = 0. */
+double orc_elen_thm3(const double* gamma, int K) {
+  double e = 0.0;
+  for (int k = 1; k <= K + 1; ++k) {
+    double gk = (k <= K) ? gamma[k - 1] : 0.0;
+    double prod = 1.0;
+    for (int j = 1; j <= k - 1; ++j) prod *= gamma[j - 1];
+    e += (double)k * (1.0 - gk) * prod;
+  }
+  return e;
+}
+
+/* Sec. 3.3 (chunk form, App. B.3): f = 1 - E_len / (K+1). */
+double orc_loss_length(double e_len, int K) { return 1.0 - e_len / (double)(K + 1); }
+
+/* App. B.3 acceptance-rate loss over a chunk of K drafted tokens:
+ * f = (1/K) sum_{j=1..K} (1 - gamma_j). */
+double orc_loss_accept(const double* gamma, int K) {
+  double s = 0.0;
+  for (int k = 0; k < K; ++k) s += 1.0 - gamma[k];
+  return s / (double)K;
+}
+
+/* ---- whole feedback call ---------------------------------------------- */
+
+/* target [B,P,V] (or, with path != NULL, a tree [B,M,V] whose rows
+ * path[b*P+k] lie on the verified path), drafter [N,B,P,V].
+ * Writes alpha [N,B,P] for every position and e_len [N,B] from
+ * alpha_1..alpha_K, K = P-1 (gamma_{K+1} := 0 in Thm 3). */
+static int feedback_impl(const void* target, const int32_t* path, int M,
+                         const void* drafter, int dtype, int N, int B, int P,
+                         int V, double T, int greedy, double* alpha,
+                         double* e_len) {
+  if (N < 1 || B < 1 || P < 1 || V < 1 || (!greedy && !(T > 0.0)))
+    return ORC_BADARG;
+  size_t esz = (dtype == ORC_FP32) ? 4 : 2;
+  int status = ORC_OK;
+  double* Pt = (double*)malloc(sizeof(double) * (size_t)V);
+  double* Q = (double*)malloc(sizeof(double) * (size_t)V);
+  for (int b = 0; b < B; ++b) {
+    for (int k = 0; k < P; ++k) {
+      int64_t trow = path ? ((int64_t)b * M + path[b * P + k]) : ((int64_t)b * P + k);
+      if (path && (path[b * P + k] < 0 || path[b * P + k] >= M)) {
+        free(Pt);
+        free(Q);
+        return ORC_BADARG;
+      }
+      const char* zt = (const char*)target + (size_t)trow * V * esz;
+      int jt = -1, st_t = ORC_OK;
+      if (greedy)
+        jt = orc_row_argmax(zt, dtype, V);
+      else
+        st_t = orc_row_probs(zt, dtype, V, T, Pt);
+      for (int i = 0; i < N; ++i) {
+        int64_t drow = ((int64_t)i * B + b) * P + k;
+        const char* zd = (const char*)drafter + (size_t)drow * V * esz;
+        double a;
+        if (greedy) {
+          int jd = orc_row_argmax(zd, dtype, V);
+          a = (jt < 0 || jd < 0) ? NAN : (jt == jd ? 1.0 : 0.0);
+        } else {
+          int st_d = orc_row_probs(zd, dtype, V, T, Q);
+          a = (st_t || st_d) ? NAN : orc_overlap(Pt, Q, V);
+        }
+        if (isnan(a)) status = ORC_NONFINITE;
+        alpha[drow] = a;
+      }
+    }
+  }
+  for (int i = 0; i < N; ++i)
+    for (int b = 0; b < B; ++b)
+      e_len[i * B + b] = orc_elen_prefix(alpha + ((size_t)i * B + b) * P, P - 1);
+  free(Pt);
+  free(Q);
+  return status;
+}
+
+int orc_feedback(const void* target, const void* drafter, int dtype, int N,
+                 int B, int P, int V, double T, int greedy, double* alpha,
+                 double* e_len) {
+  return feedback_impl(target, NULL, 0, drafter, dtype, N, B, P, V, T, greedy,
+                       alpha, e_len);
+}
+
+int orc_feedback_path(const void* tree, const int32_t* path, int M,
+                      const void* drafter, int dtype, int N, int B, int P,
+                      int V, double T, int greedy, double* alpha,
+                      double* e_len) {
+  if (M < 1 || !path) return ORC_BADARG;
+  return feedback_impl(tree, path, M, drafter, dtype, N, B, P, V, T, greedy,
+                       alpha, e_len);
+}
+
+/* ---- learners ---------------------------------------------------------- */
+
+/* Hedge (App. B.1 remark): starting from w = 1, w_i <- w_i exp(-eta l_i)
+ * after every loss vector, so w_i = exp(-eta L_i) with L the cumulative loss;
+ * Predict normalises.  exp(-eta (L_i - min L)) is the same vector up to the
+ * common factor exp(eta min L).  The played drafter is the argmax of the
+ * weights, i.e. the first argmin of L. */
+void orc_hedge(const double* L, int N, double eta, double* w, int* sel) {
+  int best = 0;
+  for (int i = 1; i < N; ++i)
+    if (L[i] < L[best]) best = i;
+  double z = 0.0;
+  for (int i = 0; i < N; ++i) {
+    w[i] = exp(-eta * (L[i] - L[best]));
+    z += w[i];
+  }
+  for (int i = 0; i < N; ++i) w[i] /= z;
+  *sel = best;
+}
+
+/* (1/N) sum_i exp(([R_i]_+)^2 / (2c)) - e : the NormalHedge scale equation. */
+static double nh_phi(const double* R, int N, double c) {
+  double s = 0.0;
+  for (int i = 0; i < N; ++i) {
+    double r = R[i] > 0.0 ? R[i] : 0.0;
+    s += exp(r * r / (2.0 * c));
+  }
+  return s / (double)N - exp(1.0);
+}
+
+/* NormalHedge, one round (App. D.6, Fig. "NormalHedge", steps 2-5).
+ * p holds p_t on entry and p_{t+1} on exit; R holds R_{t-1} / R_t.
+ * Steps 2-3 add l_A - l_i with l_A = sum_j p_j l_j.  Because sum_j p_j = 1
+ * this increment is sum_j p_j (l_j - l_i), which is how it is evaluated: the
+ * two agree to rounding, and this form is exactly 0 for a drafter whose loss
+ * ties every other's (frequent with greedy feedback, whose losses are
+ * quantised), where l_A - l_i would leave rounding noise that the scale
+ * equation then amplifies.
+ * If no regret is positive the scale equation has no root; p_{t+1} is then
+ * uniform.  The played drafter is the argmax of p_{t+1}: the first argmax of
+ * R when max R > 0 (p is strictly increasing in [R]_+ there and zero for
+ * R <= 0), else drafter 0 (uniform weights, ties to the lowest index). */
+int orc_normalhedge(double* R, const double* loss, double* p, int N, int* sel,
+                    double* c_out) {
+  for (int i = 0; i < N; ++i) {                      /* steps 2-3 */
+    double inc = 0.0;
+    for (int j = 0; j < N; ++j) inc += p[j] * (loss[j] - loss[i]);
+    R[i] += inc;
+  }
+  int best = 0;
+  for (int i = 1; i < N; ++i)
+    if (R[i] > R[best]) best = i;
+  double rmax = R[best];
+  if (!(rmax > 0.0)) {
+    for (int i = 0; i < N; ++i) p[i] = 1.0 / (double)N;
+    *sel = 0;
+    if (c_out) *c_out = NAN;
+    return ORC_OK;
+  }
+  /* step 4: phi is strictly decreasing in c; phi(lo) >= 0 because the largest
+   * term alone is N e there, phi(hi) <= 0 because every term is <= e there. */
+  double lo = rmax * rmax / (2.0 * (1.0 + log((double)N)));
+  double hi = rmax * rmax / 2.0;
+  for (int it = 0; it < 400 && (hi - lo) > 1e-15 * hi; ++it) {
+    double mid = 0.5 * (lo + hi);
+    if (nh_phi(R, N, mid) > 0.0)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  double c = 0.5 * (lo + hi);
+  double z = 0.0;                                    /* step 5 */
+  for (int i = 0; i < N; ++i) {
+    double r = R[i] > 0.0 ? R[i] : 0.0;
+    p[i] = (r / c) * exp(r * r / (2.0 * c));
+    z += p[i];
+  }
+  for (int i = 0; i < N; ++i) p[i] /= z;
+  *sel = best;
+  if (c_out) *c_out = c;
+  return ORC_OK;
+}
+
+/* One learner round for B independent queries, arrays [N,B] (element i*B+b),
+ * alpha [N,B,P], e_len [N,B].  loss_kind selects the Sec. 3.3 length loss or
+ * the acceptance-rate loss; learner_kind selects Hedge (state = cumulative
+ * loss L) or NormalHedge (state = cumulative regret R, weights = p_t in,
+ * p_{t+1} out).  selected[b] holds the drafter played this round on entry
+ * and the next round's choice on exit; when played != NULL, played[b]
+ * accumulates f_t[i_t], the learner's own loss in the Sec. 3.1 regret. */
+int orc_learner_step(const double* alpha, const double* e_len, int N, int B,
+                     int P, int loss_kind, int learner_kind, double eta,
+                     double* state, double* weights, double* loss_out,
+                     int* selected, double* played) {
+  int K = P - 1;
+  if (N < 1 || B < 1 || P < 1) return ORC_BADARG;
+  if (loss_kind == ORC_LOSS_ACCEPT && K < 1) return ORC_BADARG;
+  double* f = (double*)malloc(sizeof(double) * (size_t)N);
+  double* col = (double*)malloc(sizeof(double) * (size_t)N);
+  double* w = (double*)malloc(sizeof(double) * (size_t)N);
+  double* g = (double*)malloc(sizeof(double) * (size_t)(P > 0 ? P : 1));
+  for (int b = 0; b < B; ++b) {
+    for (int i = 0; i < N; ++i) {
+      if (loss_kind == ORC_LOSS_LENGTH) {
+        f[i] = orc_loss_length(e_len[i * B + b], K);
+      } else {
+        for (int k = 0; k < P; ++k) g[k] = alpha[((size_t)i * B + b) * P + k];
+        f[i] = orc_loss_accept(g, K);
+      }
+      if (loss_out) loss_out[i * B + b] = f[i];
+    }
+    if (played) played[b] += f[selected[b]];
+    for (int i = 0; i < N; ++i) col[i] = state[i * B + b];
+    int sel = 0;
+    if (learner_kind == ORC_HEDGE) {
+      for (int i = 0; i < N; ++i) col[i] += f[i];
+      orc_hedge(col, N, eta, w, &sel);
+    } else {
+      for (int i = 0; i < N; ++i) w[i] = weights[i * B + b];
+      orc_normalhedge(col, f, w, N, &sel, NULL);
+    }
+    for (int i = 0; i < N; ++i) {
+      state[i * B + b] = col[i];
+      weights[i * B + b] = w[i];
+    }
+    selected[b] = sel;
+  }
+  free(f);
+  free(col);
+  free(w);
+  free(g);
+  return ORC_OK;
+}

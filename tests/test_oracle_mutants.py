@@ -1,0 +1,73 @@
+"""Planted mistakes in the oracle must be caught by its pins.
+
+Each case copies ``oracle/hedgefb_oracle.c``, replaces one exact snippet by a
+plausible mistake (a dropped term, a flipped sign, a shifted or transposed
+index, a wrong tie rule), builds the copy and runs the pins against it.  The
+case passes when at least one pin fails.  CPU only.
+"""
+import os
+
+import pytest
+
+import oracle
+from oracle_pins import ALL_CHECKS
+
+MUTANTS = {
+    "overlap_max_not_min": ("a += (P[v] < Q[v]) ? P[v] : Q[v];", "a += (P[v] < Q[v]) ? Q[v] : P[v];"),
+    "tv_no_half": ("return 0.5 * t;", "return t;"),
+    "softmax_max_without_T": ("double s = orc_decode(row, dtype, v) / T;\n    if (s > m)",
+                              "double s = orc_decode(row, dtype, v);\n    if (s > m)"),
+    "softmax_sum_without_T": ("sum += exp(orc_decode(row, dtype, v) / T - m);",
+                              "sum += exp(orc_decode(row, dtype, v) - m);"),
+    "softmax_prob_without_T": ("P[v] = exp(orc_decode(row, dtype, v) / T - lse);",
+                               "P[v] = exp(orc_decode(row, dtype, v) - lse);"),
+    "lse_drops_max": ("double lse = m + log(sum);", "double lse = log(sum);"),
+    "elen_prefix_starts_at_zero": ("double e = 1.0, prod = 1.0;", "double e = 0.0, prod = 1.0;"),
+    "elen_thm3_weight_k_minus_1": ("e += (double)k * (1.0 - gk) * prod;",
+                                   "e += (double)(k - 1) * (1.0 - gk) * prod;"),
+    "elen_thm3_no_gamma_K_plus_1_zero": ("double gk = (k <= K) ? gamma[k - 1] : 0.0;",
+                                         "double gk = (k <= K) ? gamma[k - 1] : 1.0;"),
+    "loss_length_over_K": ("return 1.0 - e_len / (double)(K + 1);", "return 1.0 - e_len / (double)K;"),
+    "loss_accept_sums_gamma": ("s += 1.0 - gamma[k];", "s += gamma[k];"),
+    "hedge_sign": ("w[i] = exp(-eta * (L[i] - L[best]));", "w[i] = exp(eta * (L[i] - L[best]));"),
+    "hedge_argmax_of_loss": ("if (L[i] < L[best]) best = i;", "if (L[i] > L[best]) best = i;"),
+    "nh_regret_sign": ("inc += p[j] * (loss[j] - loss[i]);", "inc += p[j] * (loss[i] - loss[j]);"),
+    "nh_learner_loss_unweighted": ("inc += p[j] * (loss[j] - loss[i]);",
+                                   "inc += (loss[j] - loss[i]) / (double)N;"),
+    "nh_weight_drops_r_over_c": ("p[i] = (r / c) * exp(r * r / (2.0 * c));", "p[i] = exp(r * r / (2.0 * c));"),
+    "nh_equation_c_not_2c": ("s += exp(r * r / (2.0 * c));", "s += exp(r * r / c);"),
+    "nh_uniform_branch_picks_argmax": ("p[i] = 1.0 / (double)N;\n    *sel = 0;",
+                                       "p[i] = 1.0 / (double)N;\n    *sel = best;"),
+    "argmax_last_on_ties": ("if (z > bz) { bz = z; best = v; }", "if (z >= bz) { bz = z; best = v; }"),
+    "bf16_shift_15": ("((uint32_t)h) << 16;", "((uint32_t)h) << 15;"),
+    "fp16_bias": ("expo - 25);", "expo - 24);"),
+    "nonfinite_misses_inf": ("if (isnan(z) || z == INFINITY) return 0;", "if (isnan(z)) return 0;"),
+    "drafter_index_transposed": ("int64_t drow = ((int64_t)i * B + b) * P + k;",
+                                 "int64_t drow = ((int64_t)b * N + i) * P + k;"),
+    "target_index_transposed": ("((int64_t)b * P + k);", "((int64_t)k * B + b);"),
+    "elen_uses_all_P_positions": ("* P, P - 1);", "* P, P);"),
+    "greedy_inverted": ("a = (jt < 0 || jd < 0) ? NAN : (jt == jd ? 1.0 : 0.0);",
+                        "a = (jt < 0 || jd < 0) ? NAN : (jt != jd ? 1.0 : 0.0);"),
+    "played_loss_wrong_drafter": ("played[b] += f[selected[b]];", "played[b] += f[0];"),
+    "hedge_state_not_cumulative": ("for (int i = 0; i < N; ++i) col[i] += f[i];",
+                                   "for (int i = 0; i < N; ++i) col[i] = f[i];"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    with open(oracle._SRC) as f:
+        src = f.read()
+    assert src.count(old) == 1, f"snippet for {name} must occur exactly once"
+    mpath = os.path.join(tmp_path, "mutant.c")
+    with open(mpath, "w") as f:
+        f.write(src.replace(old, new))
+    lib = oracle.build(mpath, os.path.join(tmp_path, f"libmutant_{name}.so"))
+    o = oracle.Oracle(lib)
+    for check in ALL_CHECKS:
+        try:
+            check(o)
+        except AssertionError:
+            return
+    pytest.fail(f"no pin caught the planted mistake {name}")
