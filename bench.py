@@ -1,0 +1,446 @@
+#!/usr/bin/env python3
+"""Benchmark of the HedgeSpec panoramic-feedback step on GB300.
+
+One step = hs_feedback (alpha and e_len for every drafter, query and
+position) + hs_learner_step (length loss, NormalHedge or Hedge update and
+the next choice) on one batch of seeded synthetic logits already resident in
+HBM.  Prints ONE JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                  [--mode stochastic|greedy] [--impl ours|reference]
+
+Timing: the K steps run as CUDA-graph replays on one stream, bracketed by
+CUDA events after a barrier + synchronize; inputs rotate over enough buffer
+sets (>= 2x the L2 size in total) that no call finds its logits in L2.  The
+feedback path alone is timed the same way in a second region for the
+roofline.  `e2e` repeats the step through the public API from pinned host
+buffers, with the host->device copy of every step's logits and the
+device->host read of its result (weights and choice) inside the timed region.
+Under torchrun each rank runs its own queries (weak scaling, no collective on
+the data path); value = all ranks' evaluations / the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("drafter-position-vocab evals/s and achieved HBM GB/s (% of GB300 peak) "
+          "per hs_feedback")
+DEFAULT_WORKLOAD = "qwen3_8b_chain"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--mode", choices=("stochastic", "greedy"), default="stochastic")
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    return ap.parse_args()
+
+
+# ---- distributed plumbing ---------------------------------------------------
+
+def dist_info():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def dist_init(world, backend):
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+
+
+def barrier(world, device=None):
+    if world > 1:
+        import torch.distributed as dist
+        if device is not None:
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---- clocks during the timed region -----------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", self.gpu_id], stdout=self.out, stderr=subprocess.DEVNULL)
+            self.t0 = time.time()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        if time.time() - self.t0 < 0.35:
+            time.sleep(0.35 - (time.time() - self.t0))
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for _, _, flags in rows for j, v in enumerate(flags)
+                          if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+def gpu_uuid(dev) -> str:
+    import torch
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return str(dev.index)
+
+
+# ---- roofline inputs ----------------------------------------------------------
+
+def measured_hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2510_20064_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str, mode: str):
+    """DRAM bytes per feedback call from a committed ncu summary, if that
+    summary was taken on the current kernel sources."""
+    path = os.path.join(ROOT, "profiles", f"feedback_{workload}_{mode}.md")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line and line.strip().startswith("- "):
+                k, v = line.strip()[2:].split(":", 1)
+                fields[k.strip()] = v.strip().strip("`")
+    if fields.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    try:
+        return int(fields["dram_bytes_per_call"])
+    except (KeyError, ValueError):
+        return None
+
+
+# ---- CPU oracle baseline ------------------------------------------------------
+
+def oracle_sample(w, sets, greedy, budget_s=10.0):
+    """The fp64 C oracle (single-threaded, as it stands) on whole (b,k)
+    tiles of the first input set until ~budget_s seconds of CPU work."""
+    import oracle
+    from paper_2510_20064_gb300 import synth
+    o = oracle.get()
+    d = sets[0]
+    t_all = synth.storage_numpy(d["target"])
+    path = d.get("path")
+    path_np = None if path is None else path.cpu().numpy()
+    evals, tiles, t_used = 0, 0, 0.0
+    tile = 0
+    while t_used < budget_s and tile < w.B * w.P:
+        b, k = divmod(tile, w.P)
+        trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
+        drows = synth.storage_numpy(d["drafter"][:, b, k])
+        t0 = time.perf_counter()
+        for i in range(w.N):
+            o.alpha_pair(trow, drows[i], w.temperature, greedy)
+        t_used += time.perf_counter() - t0
+        evals += w.N * w.V
+        tiles += 1
+        tile += 1
+    return {"value": evals / t_used, "unit": "evals/s", "cores": 1, "kind": "oracle",
+            "sample": f"{tiles} of {w.B * w.P} (b,k) tiles x {w.N} drafters x V={w.V} of the "
+                      f"{w.name} workload, fp64 C oracle, 1 thread, {t_used:.1f} s"}
+
+
+# ---- the benchmark -------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+
+    import paper_2510_20064_gb300 as hf
+    from paper_2510_20064_gb300 import synth
+
+    rank, world, local = dist_info()
+    assert torch.cuda.is_available(), "bench.py needs a GPU"
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    dist_init(world, "nccl")
+    hf.lib()
+
+    w = synth.WORKLOADS[args.workload]
+    greedy = args.mode == "greedy"
+    learner = hf.HS_HEDGE if w.learner == "hedge" else hf.HS_NORMALHEDGE
+    N, B, P, V = w.N, w.B, w.P, w.V
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 129 * 2**20
+    n_sets = max(2, math.ceil(2 * l2 / w.bytes_per_call))
+    sets = [synth.make_inputs(w, rnd=s, device=dev, seed=w.seed_base + 100000 * rank + s)
+            for s in range(n_sets)]
+
+    stream = torch.cuda.Stream(device=dev)
+    alpha = torch.empty(N, B, P, device=dev)
+    e_len = torch.empty(N, B, device=dev)
+    ws_bytes = hf.hs_feedback_workspace_size(N, B, P, V, synth.DTYPES[w.dtype], greedy)
+    ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    state = torch.zeros(N, B, device=dev)
+    weights = torch.full((N, B), 1.0 / N, device=dev)
+    sel = torch.zeros(B, dtype=torch.int32, device=dev)
+    eta = w.eta if w.eta else math.sqrt(8 * math.log(max(N, 2)) / 2000)
+
+    def feedback(d):
+        if "path" in d:
+            hf.hs_feedback_path(d["target"], d["path"], d["drafter"], w.temperature, greedy,
+                                alpha=alpha, e_len=e_len, workspace=ws, dev_status=status,
+                                stream=stream)
+        else:
+            hf.hs_feedback(d["target"], d["drafter"], w.temperature, greedy, alpha=alpha,
+                           e_len=e_len, workspace=ws, dev_status=status, stream=stream)
+
+    def step(d):
+        feedback(d)
+        hf.hs_learner_step(alpha, e_len, hf.HS_LOSS_LENGTH, learner, eta, state, weights, sel,
+                           stream=stream)
+
+    # eager warm-up, then graphs of whole steps and of feedback calls
+    with torch.cuda.stream(stream):
+        for s in range(max(args.warmup, 3)):
+            step(sets[s % n_sets])
+    stream.synchronize()
+    per_graph = n_sets * max(1, math.ceil(32 / n_sets))
+
+    def capture(fn, count):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for s in range(count):
+                fn(sets[s % n_sets])
+        return g
+
+    def timed(fn, steps):
+        full, rem = divmod(steps, per_graph)
+        g_full = capture(fn, per_graph) if full else None
+        g_rem = capture(fn, rem) if rem else None
+        for _ in range(2):  # graph warm-up
+            (g_full or g_rem).replay()
+        stream.synchronize()
+        barrier(world, dev)
+        torch.cuda.synchronize(dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(full):
+            g_full.replay()
+        if rem:
+            g_rem.replay()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(world, dev)
+        return t0.elapsed_time(t1) / 1e3
+
+    clocks = ClockSampler(gpu_uuid(dev))
+    clocks.start()
+    t_step = timed(step, args.steps)
+    clk = clocks.stop()
+    t_fb = timed(feedback, args.steps)
+    assert int(status.item()) == 0, hf.hs_status_string(int(status.item()))
+
+    # ---- end to end through the public API from pinned host buffers ----
+    host_sets = [{k: v.cpu().pin_memory() for k, v in d.items() if torch.is_tensor(v)}
+                 for d in sets[:2]]
+    dsts = {k: torch.empty_like(v, device=dev) for k, v in host_sets[0].items()}
+    out_w = torch.empty(N, B).pin_memory()
+    out_s = torch.empty(B, dtype=torch.int32).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for k, v in host_sets[0].items() if k != "sigma")
+    d2h = out_w.numel() * 4 + out_s.numel() * 4
+    e2e_steps = max(1, min(args.steps, args.e2e_steps))
+    with torch.cuda.stream(stream):
+        barrier(world, dev)
+        torch.cuda.synchronize(dev)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(e2e_steps):
+            hs = host_sets[s % 2]
+            for k, v in hs.items():
+                if k != "sigma":
+                    dsts[k].copy_(v, non_blocking=True)
+            step(dsts)
+            out_w.copy_(weights, non_blocking=True)
+            out_s.copy_(sel, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+    t_e2e = e0.elapsed_time(e1) / 1e3
+
+    t_step = max_over_ranks(t_step, world, dev)
+    t_fb = max_over_ranks(t_fb, world, dev)
+    t_e2e = max_over_ranks(t_e2e, world, dev)
+    evals_step = w.evals
+    value = world * args.steps * evals_step / t_step
+    peak, peak_src = measured_hbm_peak()
+    fb_avg = t_fb / args.steps
+    achieved = w.bytes_per_call / fb_avg / 1e9
+    launches_step = hf.hs_feedback_kernel_count(N, B, P, V, synth.DTYPES[w.dtype], greedy) + 1
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = oracle_sample(w, sets, greedy)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * t_step / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic: seeded Zipf + Gaussian logits, drafter = target + noise "
+                    "(no dataset, no trained weights)",
+            "config": {"workload": w.name, "N": N, "B": B, "K": w.K, "V": V,
+                       "temperature": None if greedy else w.temperature, "mode": args.mode,
+                       "learner": "hedge" if learner == hf.HS_HEDGE else "normalhedge",
+                       "loss": "length", "l2": f"{n_sets} rotating input sets "
+                       f"({n_sets * w.bytes_per_call / 2**20:.0f} MiB > 2x L2 {l2 / 2**20:.0f} MiB)",
+                       "parallelism": f"queries sharded over {world} rank(s), no collective"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "peak_source": peak_src,
+                         "traffic": profiled_traffic(w.name, args.mode),
+                         "kernel": "hs_feedback (all its kernels), timed alone",
+                         "algorithmic_bytes_per_call": w.bytes_per_call,
+                         "us_per_call": 1e6 * fb_avg},
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * e2e_steps * evals_step / t_e2e, "unit": "evals/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "gpu_launches": launches_step * args.steps,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The fp64 CPU oracle on the host cores, same metric and config."""
+    rank, world, _ = dist_info()
+    if rank != 0:
+        return
+    import oracle
+    import torch
+    from paper_2510_20064_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    greedy = args.mode == "greedy"
+    d = synth.make_inputs(w, device="cpu", B=min(w.B, 2))
+    o = oracle.get()
+    t_all = synth.storage_numpy(d["target"])
+    path = d.get("path")
+    path_np = None if path is None else path.numpy()
+    tiles = [(b, k) for b in range(d["drafter"].shape[1]) for k in range(w.P)]
+
+    def one(s):
+        b, k = tiles[s % len(tiles)]
+        trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
+        drows = synth.storage_numpy(d["drafter"][:, b, k])
+        for i in range(w.N):
+            o.alpha_pair(trow, drows[i], w.temperature, greedy)
+
+    for s in range(args.warmup):
+        one(s)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        one(s)
+    t = time.perf_counter() - t0
+    value = args.steps * w.N * w.V / t
+    sample = (f"each step = one (b,k) tile of {w.name}: {w.N} drafter rows x V={w.V}, "
+              "fp64 C oracle, 1 thread")
+    del torch
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "evals/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "N": w.N, "B": w.B, "K": w.K, "V": w.V,
+                   "mode": args.mode},
+        "cpu_baseline": {"value": value, "unit": "evals/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "evals/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,175 @@
+/*
+ * hedgefb.h -- C ABI of libhedgefb, the GB300 (sm_103a) implementation of
+ * HedgeSpec's panoramic-feedback path ("Not-a-Bandit: Provably No-Regret
+ * Drafter Selection in Speculative Decoding for LLMs", arXiv 2510.20064).
+ *
+ * After a verification step the verified tokens have been prefilled into
+ * every drafter (Sec. 3.2), so each drafter i has logits at the same P = K+1
+ * positions as the target.  From those logits this library computes
+ *   alpha[i,b,k] -- the token acceptance probability gamma (Sec. 3.2):
+ *                   sum_v min(p(v), q_i(v)) (Thm 1), or, in greedy mode, the
+ *                   indicator that argmax q_i == argmax p (Thm 2, L = 1);
+ *   e_len[i,b]   -- the acceptance-length estimate of Thm 3,
+ *                   1 + sum_{k=1..K} prod_{j<=k} alpha_j, with gamma_{K+1} = 0;
+ * and then runs the learner: the Sec. 3.3 loss, Hedge (App. B.1 remark) or
+ * NormalHedge (App. D.6 figure), and the choice of the next drafter.
+ *
+ * Conventions shared by every call
+ *  - Shapes are row-major and contiguous.  Index names: N drafters, B
+ *    queries, P = K+1 positions, V vocabulary entries.  [N,B] arrays hold
+ *    element (i,b) at i*B + b.
+ *  - Every pointer marked "device" is device memory owned by the caller; the
+ *    library allocates nothing and keeps no state between calls.
+ *  - Logits are bf16, fp16 or fp32 (hs_dtype); probabilities, losses, state
+ *    and weights are fp32; indices are int32.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream).  Argument errors are detected on the host, before any
+ *    launch, and returned; nothing is launched then.  HS_ERR_CUDA reports a
+ *    failed launch (cudaGetLastError).
+ *  - Data errors are found on the device.  A logit row holding NaN or +inf,
+ *    or holding only -inf, makes every alpha that uses the row NaN (and the
+ *    e_len that uses it); then, if dev_status is not NULL, HS_ERR_NONFINITE
+ *    is stored to *dev_status.  An out-of-range path index stores
+ *    HS_ERR_INVALID_ARG the same way.  The library never clears *dev_status:
+ *    set it to HS_OK before the call and read it after synchronising.
+ *    -inf logits are legal (masked vocabulary).
+ *  - Nothing traps; no kernel waits without a bound.
+ */
+#ifndef HEDGEFB_H
+#define HEDGEFB_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  HS_OK = 0,
+  HS_ERR_INVALID_ARG = 1,  /* bad size, null pointer, T <= 0, short workspace */
+  HS_ERR_UNSUPPORTED = 2,  /* well-formed but outside what is built (e.g. N > 32 for a learner) */
+  HS_ERR_MISALIGNED = 3,   /* a pointer not aligned to its element type */
+  HS_ERR_NONFINITE = 4,    /* device-side: NaN / +inf / all -inf logit row */
+  HS_ERR_CUDA = 5,         /* a CUDA launch failed */
+  HS_ERR_TIMEOUT = 6       /* device-side: a bounded wait ran out */
+} hs_status;
+
+typedef enum { HS_BF16 = 0, HS_FP16 = 1, HS_FP32 = 2 } hs_dtype;
+typedef enum { HS_LOSS_LENGTH = 0, HS_LOSS_ACCEPT = 1 } hs_loss;
+typedef enum { HS_HEDGE = 0, HS_NORMALHEDGE = 1 } hs_learner;
+
+/* Largest N the learner calls accept (one warp lane per drafter). */
+#define HS_MAX_LEARNER_N 32
+
+/* Human-readable name of a status code; never NULL. */
+const char* hs_status_string(int status);
+
+/* Library version, 10000*major + 100*minor + patch. */
+int hs_version(void);
+
+/* Bytes of device workspace hs_feedback / hs_feedback_path need for these
+ * sizes (0 is a valid answer).  Returns 0 for invalid sizes as well; those
+ * calls then fail with HS_ERR_INVALID_ARG. */
+size_t hs_feedback_workspace_size(int N, int B, int P, int V, int dtype, int greedy);
+
+/* Number of kernels one hs_feedback / hs_feedback_path call with these
+ * arguments launches (for launch accounting); 0 for invalid sizes. */
+int hs_feedback_kernel_count(int N, int B, int P, int V, int dtype, int greedy);
+
+/* Panoramic feedback along a verified chain (Sec. 3.2; Thm 1, Thm 2 with
+ * L = 1, Thm 3).
+ *   target     device, [B,P,V] logits of the target at the P = K+1 verified
+ *              positions (Sec. 2.2 step 2: p(x_{t+k} | x_{<t+k}), k = 1..K+1).
+ *   drafter    device, [N,B,P,V] logits of every drafter prefilled with the
+ *              same verified tokens (Sec. 3.2).
+ *   dtype      hs_dtype of both logit tensors.
+ *   temperature  T > 0, finite: p = softmax(z_target / T), q_i =
+ *              softmax(z_i / T).  Ignored when greedy != 0.
+ *   greedy     0: alpha = sum_v min(p(v), q_i(v)), fp32 accumulation.
+ *              1: alpha = 1 if argmax q_i == argmax p else 0, argmax over the
+ *                 stored logits, lowest index on ties (exact).
+ *   alpha      device, out, [N,B,P] fp32 -- all P positions.  The last one
+ *              (k = K+1) is the first position of the next chunk; it is not
+ *              used by e_len (gamma_{K+1} := 0 in Thm 3).
+ *   e_len      device, out, [N,B] fp32 -- 1 + sum_{k=1..K} prod_{j<=k} alpha_j,
+ *              in [1, K+1].  May be NULL.
+ *   workspace  device, hs_feedback_workspace_size(...) bytes, 256-byte
+ *              aligned; may be NULL when that size is 0.  Its contents need
+ *              no initialisation and are garbage afterwards.
+ *   dev_status device, one int, or NULL (see conventions).
+ * Limits: N, B, P, V >= 1; N*B*P*V < 2^62.  Misaligned logit pointers (not
+ * a multiple of the element size) give HS_ERR_MISALIGNED. */
+hs_status hs_feedback(const void* target, const void* drafter, int dtype, int N,
+                      int B, int P, int V, float temperature, int greedy,
+                      float* alpha, float* e_len, void* workspace,
+                      size_t workspace_bytes, int* dev_status, void* stream);
+
+/* As hs_feedback, but the target rows come from a draft tree (Sec. 2.3,
+ * Fig. "illus_gamma"): row k of query b is tree_target[b, path_idx[b,k], :].
+ *   tree_target  device, [B,M,V] logits at the M tree nodes of each query.
+ *   path_idx     device, [B,P] int32 node indices of the verified
+ *                root-to-leaf path, each in [0, M).  An index outside that
+ *                range makes the alphas of that (b,k) NaN and stores
+ *                HS_ERR_INVALID_ARG to *dev_status.
+ * Only the P path rows of each query are read. */
+hs_status hs_feedback_path(const void* tree_target, const int32_t* path_idx,
+                           int M, const void* drafter, int dtype, int N, int B,
+                           int P, int V, float temperature, int greedy,
+                           float* alpha, float* e_len, void* workspace,
+                           size_t workspace_bytes, int* dev_status,
+                           void* stream);
+
+/* Hedge weights from cumulative losses (App. B.1 remark: w_i <- w_i
+ * exp(-eta l_i) from w = 1, normalised, i.e. w = exp(-eta L) / Z).
+ *   cum_loss  device, [N,B] fp32 cumulative loss L per (drafter, query).
+ *   eta       learning rate, finite and >= 0.
+ *   weights   device, out, [N,B] fp32, each column sums to 1.
+ *   selected  device, out, [B] int32: first argmin_i L[i,b] (= argmax of w).
+ * Limits: 1 <= N <= HS_MAX_LEARNER_N, B >= 1. */
+hs_status hs_hedge_update(const float* cum_loss, int N, int B, float eta,
+                          float* weights, int32_t* selected, void* stream);
+
+/* One NormalHedge round (App. D.6 figure, steps 2-5) for B queries.
+ *   regret    device, in/out, [N,B] fp32: R_{t-1} in, R_t out, where
+ *             R_t = R_{t-1} + l_A - l evaluated as sum_j p_j (l_j - l_i).
+ *   loss      device, [N,B] fp32 losses l_t of this round.
+ *   weights   device, in/out, [N,B] fp32: p_t in (initially 1/N), p_{t+1}
+ *             out: p_i proportional to ([R_i]_+/c) exp([R_i]_+^2 / 2c) with
+ *             c solving (1/N) sum_i exp([R_i]_+^2 / 2c) = e; uniform when no
+ *             R_i is positive.
+ *   selected  device, out, [B] int32: argmax of p_{t+1} -- the first argmax
+ *             of R when max R > 0, else 0.
+ * Limits: 1 <= N <= HS_MAX_LEARNER_N, B >= 1. */
+hs_status hs_normalhedge_update(float* regret, const float* loss,
+                                float* weights, int N, int B,
+                                int32_t* selected, void* stream);
+
+/* Fused learner round: loss from the feedback (Sec. 3.3), learner update and
+ * next choice, for B independent queries.
+ *   alpha, e_len  device, [N,B,P] and [N,B] fp32 from hs_feedback.
+ *   loss_kind     HS_LOSS_LENGTH: f = 1 - e_len / (K+1)      (needs e_len)
+ *                 HS_LOSS_ACCEPT: f = (1/K) sum_{k<=K} (1 - alpha_k)
+ *                                 (needs alpha and P >= 2)
+ *   learner       HS_HEDGE:       state = cumulative loss L, L += f, then
+ *                                 hs_hedge_update's weights and choice
+ *                 HS_NORMALHEDGE: state = cumulative regret R, then
+ *                                 hs_normalhedge_update's round
+ *   eta           Hedge learning rate (ignored by NormalHedge).
+ *   state, weights  device, in/out, [N,B] fp32.
+ *   loss_out      device, out, [N,B] fp32 losses f, or NULL.
+ *   selected      device, in/out, [B] int32: the drafter played this round
+ *                 in, the next round's choice out.
+ *   played_loss   device, in/out, [B] fp32, or NULL: += f[selected_in],
+ *                 the learner's own loss term of the Sec. 3.1 regret.
+ * Limits: 1 <= N <= HS_MAX_LEARNER_N, B >= 1, P >= 1. */
+hs_status hs_learner_step(const float* alpha, const float* e_len, int N, int B,
+                          int P, int loss_kind, int learner, float eta,
+                          float* state, float* weights, float* loss_out,
+                          int32_t* selected, float* played_loss, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HEDGEFB_H */

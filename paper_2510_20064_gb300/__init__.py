@@ -1,0 +1,221 @@
+"""Python binding of libhedgefb (HedgeSpec panoramic feedback on GB300).
+
+Argument marshalling only: every entry point checks the tensors it is given
+(device, dtype, shape, contiguity), allocates missing outputs with torch and
+passes raw pointers to the C ABI declared in ``include/hedgefb.h``.  All
+arithmetic runs in the library's CUDA kernels; there is no other code path.
+Importing this module fails loudly when ``libhedgefb.so`` has not been built
+(``python -m paper_2510_20064_gb300.build`` or ``__graft_entry__.build()``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libhedgefb.so")
+
+HS_OK, HS_ERR_INVALID_ARG, HS_ERR_UNSUPPORTED, HS_ERR_MISALIGNED = 0, 1, 2, 3
+HS_ERR_NONFINITE, HS_ERR_CUDA, HS_ERR_TIMEOUT = 4, 5, 6
+HS_BF16, HS_FP16, HS_FP32 = 0, 1, 2
+HS_LOSS_LENGTH, HS_LOSS_ACCEPT = 0, 1
+HS_HEDGE, HS_NORMALHEDGE = 0, 1
+HS_MAX_LEARNER_N = 32
+
+_DTYPES = {torch.bfloat16: HS_BF16, torch.float16: HS_FP16, torch.float32: HS_FP32}
+
+# argument/return types of every exported symbol (mirrors include/hedgefb.h)
+_P, _I, _F, _Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+SIGNATURES = {
+    "hs_status_string": ([_I], ctypes.c_char_p),
+    "hs_version": ([], _I),
+    "hs_feedback_workspace_size": ([_I, _I, _I, _I, _I, _I], _Z),
+    "hs_feedback_kernel_count": ([_I, _I, _I, _I, _I, _I], _I),
+    "hs_feedback": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
+    "hs_feedback_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
+    "hs_hedge_update": ([_P, _I, _I, _F, _P, _P, _P], _I),
+    "hs_normalhedge_update": ([_P, _P, _P, _I, _I, _P, _P], _I),
+    "hs_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P], _I),
+}
+
+
+class HedgeFBError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {hs_status_string(status)}")
+
+
+_lib = None
+
+
+def lib():
+    """The loaded ``libhedgefb.so`` (ctypes), with argument types set."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(
+                f"libhedgefb.so is missing at {LIB_PATH}: build it with "
+                "`python -m paper_2510_20064_gb300.build` (needs nvcc); there is no fallback")
+        handle = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in SIGNATURES.items():
+            fn = getattr(handle, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = handle
+    return _lib
+
+
+def hs_status_string(status: int) -> str:
+    return lib().hs_status_string(int(status)).decode()
+
+
+def hs_version() -> int:
+    return lib().hs_version()
+
+
+def _check(status: int, where: str):
+    if status != HS_OK:
+        raise HedgeFBError(status, where)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if isinstance(stream, torch.cuda.Stream) else int(stream))
+
+
+def _need(t: torch.Tensor, name: str, dtype=None, shape=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype not in _DTYPES:
+        raise ValueError(f"logits must be bf16, fp16 or fp32, got {t.dtype}")
+    return _DTYPES[t.dtype]
+
+
+def hs_feedback_workspace_size(N: int, B: int, P: int, V: int, dtype, greedy: bool) -> int:
+    code = dtype if isinstance(dtype, int) else _DTYPES[dtype]
+    return int(lib().hs_feedback_workspace_size(N, B, P, V, code, int(bool(greedy))))
+
+
+def hs_feedback_kernel_count(N: int, B: int, P: int, V: int, dtype, greedy: bool) -> int:
+    code = dtype if isinstance(dtype, int) else _DTYPES[dtype]
+    return int(lib().hs_feedback_kernel_count(N, B, P, V, code, int(bool(greedy))))
+
+
+def _feedback_outputs(drafter, alpha, e_len, workspace, greedy):
+    N, B, P, V = drafter.shape
+    dev = drafter.device
+    if alpha is None:
+        alpha = torch.empty((N, B, P), device=dev, dtype=torch.float32)
+    if e_len is None:
+        e_len = torch.empty((N, B), device=dev, dtype=torch.float32)
+    _need(alpha, "alpha", torch.float32, (N, B, P))
+    _need(e_len, "e_len", torch.float32, (N, B))
+    ws_bytes = hs_feedback_workspace_size(N, B, P, V, drafter.dtype, greedy)
+    if workspace is None and ws_bytes > 0:
+        workspace = torch.empty(ws_bytes, device=dev, dtype=torch.uint8)
+    return alpha, e_len, workspace, ws_bytes
+
+
+def hs_feedback(target: torch.Tensor, drafter: torch.Tensor, temperature: float = 1.0,
+                greedy: bool = False, alpha=None, e_len=None, workspace=None,
+                dev_status=None, stream=None):
+    """alpha [N,B,P] and e_len [N,B] (fp32) from target [B,P,V] and drafter
+    [N,B,P,V] logits (Thm 1 / Thm 2 with L = 1, Thm 3)."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(target, "target", drafter.dtype, (B, P, V))
+    alpha, e_len, workspace, ws_bytes = _feedback_outputs(drafter, alpha, e_len, workspace, greedy)
+    st = lib().hs_feedback(_ptr(target), _ptr(drafter), _dtype_code(drafter), N, B, P, V,
+                           float(temperature), int(bool(greedy)), _ptr(alpha), _ptr(e_len),
+                           _ptr(workspace), ws_bytes if workspace is not None else 0,
+                           _ptr(dev_status), _stream(stream))
+    _check(st, "hs_feedback")
+    return alpha, e_len
+
+
+def hs_feedback_path(tree_target: torch.Tensor, path_idx: torch.Tensor, drafter: torch.Tensor,
+                     temperature: float = 1.0, greedy: bool = False, alpha=None, e_len=None,
+                     workspace=None, dev_status=None, stream=None):
+    """As hs_feedback with target row (b,k) = tree_target[b, path_idx[b,k]]."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(tree_target, "tree_target", drafter.dtype)
+    if tree_target.dim() != 3 or tree_target.shape[0] != B or tree_target.shape[2] != V:
+        raise ValueError(f"tree_target must be [B, M, V] = [{B}, M, {V}]")
+    M = tree_target.shape[1]
+    _need(path_idx, "path_idx", torch.int32, (B, P))
+    alpha, e_len, workspace, ws_bytes = _feedback_outputs(drafter, alpha, e_len, workspace, greedy)
+    st = lib().hs_feedback_path(_ptr(tree_target), _ptr(path_idx), M, _ptr(drafter),
+                                _dtype_code(drafter), N, B, P, V, float(temperature),
+                                int(bool(greedy)), _ptr(alpha), _ptr(e_len), _ptr(workspace),
+                                ws_bytes if workspace is not None else 0, _ptr(dev_status),
+                                _stream(stream))
+    _check(st, "hs_feedback_path")
+    return alpha, e_len
+
+
+def hs_hedge_update(cum_loss: torch.Tensor, eta: float, weights=None, selected=None, stream=None):
+    """Hedge weights exp(-eta L)/Z and first argmin of L, per query."""
+    _need(cum_loss, "cum_loss", torch.float32)
+    N, B = cum_loss.shape
+    if weights is None:
+        weights = torch.empty_like(cum_loss)
+    if selected is None:
+        selected = torch.empty(B, device=cum_loss.device, dtype=torch.int32)
+    _need(weights, "weights", torch.float32, (N, B))
+    _need(selected, "selected", torch.int32, (B,))
+    _check(lib().hs_hedge_update(_ptr(cum_loss), N, B, float(eta), _ptr(weights),
+                                 _ptr(selected), _stream(stream)), "hs_hedge_update")
+    return weights, selected
+
+
+def hs_normalhedge_update(regret: torch.Tensor, loss: torch.Tensor, weights: torch.Tensor,
+                          selected=None, stream=None):
+    """One NormalHedge round in place on (regret, weights)."""
+    _need(regret, "regret", torch.float32)
+    N, B = regret.shape
+    _need(loss, "loss", torch.float32, (N, B))
+    _need(weights, "weights", torch.float32, (N, B))
+    if selected is None:
+        selected = torch.empty(B, device=regret.device, dtype=torch.int32)
+    _need(selected, "selected", torch.int32, (B,))
+    _check(lib().hs_normalhedge_update(_ptr(regret), _ptr(loss), _ptr(weights), N, B,
+                                       _ptr(selected), _stream(stream)), "hs_normalhedge_update")
+    return regret, weights, selected
+
+
+def hs_learner_step(alpha: torch.Tensor, e_len: torch.Tensor, loss_kind: int, learner: int,
+                    eta: float, state: torch.Tensor, weights: torch.Tensor,
+                    selected: torch.Tensor, loss_out=None, played_loss=None, stream=None):
+    """Fused loss + learner round in place on (state, weights, selected)."""
+    _need(alpha, "alpha", torch.float32)
+    N, B, P = alpha.shape
+    _need(e_len, "e_len", torch.float32, (N, B))
+    _need(state, "state", torch.float32, (N, B))
+    _need(weights, "weights", torch.float32, (N, B))
+    _need(selected, "selected", torch.int32, (B,))
+    if loss_out is not None:
+        _need(loss_out, "loss_out", torch.float32, (N, B))
+    if played_loss is not None:
+        _need(played_loss, "played_loss", torch.float32, (B,))
+    _check(lib().hs_learner_step(_ptr(alpha), _ptr(e_len), N, B, P, int(loss_kind), int(learner),
+                                 float(eta), _ptr(state), _ptr(weights), _ptr(loss_out),
+                                 _ptr(selected), _ptr(played_loss), _stream(stream)),
+           "hs_learner_step")
+    return state, weights, selected

@@ -1,0 +1,389 @@
+// hs_feedback.cu -- panoramic feedback: alpha[N,B,P] and e_len[N,B].
+//
+// Two-pass path, used for greedy mode (where it reads every logit once) and
+// for stochastic rows that the fused cluster kernel does not take:
+//   row_stats_kernel  one CTA per logit row: max, first argmax and
+//                     S = sum_v 2^{(z_v - m) log2e / T}   (Thm 1's softmax)
+//   overlap_kernel    one CTA per ((b,k) tile, vocab chunk): p_v built once
+//                     and reused for all N drafters, sum_v min(p_v, q_{i,v})
+//                     (Thm 1), one partial sum per chunk
+//   finalize_kernel   one thread per (i,b): alpha over the P positions from
+//                     the partials (fixed order) or from the argmaxes
+//                     (greedy, Thm 2 with L = 1), then e_len (Thm 3).
+#include <math.h>
+#include <stdint.h>
+
+#include <climits>
+
+#include "hs_common.cuh"
+
+namespace hs {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kUnroll = 4;  // 16-byte vectors per thread per chunk
+
+// argmax < 0 marks a row that cannot be used: -1 non-finite, -2 bad path.
+struct RowStat {
+  float m;      // max of the stored logits
+  float mc;     // m * log2e / T, the exponent offset used for the row
+  float inv_s;  // 1 / sum_v 2^{z_v c - mc}
+  int argmax;   // first index of m
+};
+
+template <int DT>
+__device__ __forceinline__ const void* row_ptr(const void* base, int64_t row, int V) {
+  return static_cast<const char*>(base) + row * int64_t(V) * Elem<DT>::kBytes;
+}
+
+// Target row of tile (b,k): a chain row, or the path node of a tree.
+template <int DT>
+__device__ __forceinline__ const void* target_row(const void* target, const int32_t* path,
+                                                  int M, int P, int64_t tile, int V,
+                                                  bool* bad_path) {
+  if (!path) return row_ptr<DT>(target, tile, V);
+  int64_t b = tile / P;
+  int node = path[tile];
+  *bad_path = node < 0 || node >= M;
+  if (*bad_path) node = 0;
+  return row_ptr<DT>(target, b * M + node, V);
+}
+
+// Element v handled by slot s of thread t in a chunk starting at v0.
+template <int DT, bool VEC>
+__device__ __forceinline__ int64_t slot_pos(int64_t v0, int s, int t) {
+  constexpr int kV = Elem<DT>::kVec;
+  if (VEC) return v0 + (int64_t((s / kV) * kThreads + t)) * kV + (s % kV);
+  return v0 + int64_t(s) * kThreads + t;
+}
+
+// Load the chunk slots of one row into x[] (-inf past the end of the row).
+template <int DT, bool VEC>
+__device__ __forceinline__ void load_slots(const void* row, int64_t v0, int V,
+                                           float (&x)[kUnroll * Elem<DT>::kVec]) {
+  constexpr int kV = Elem<DT>::kVec;
+  const int t = threadIdx.x;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    if (VEC) {
+      int64_t v = v0 + int64_t(u * kThreads + t) * kV;
+      float tmp[kV];
+      if (v < V) {
+        Elem<DT>::vec(row, v, tmp);
+      } else {
+#pragma unroll
+        for (int e = 0; e < kV; ++e) tmp[e] = -INFINITY;
+      }
+#pragma unroll
+      for (int e = 0; e < kV; ++e) x[u * kV + e] = tmp[e];
+    } else {
+#pragma unroll
+      for (int e = 0; e < kV; ++e) {
+        int64_t v = slot_pos<DT, false>(v0, u * kV + e, t);
+        x[u * kV + e] = v < V ? Elem<DT>::one(row, v) : -INFINITY;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < kWarps; ++j) s += red[j];
+  return s;
+}
+
+template <int DT, bool VEC, bool GREEDY>
+__global__ void __launch_bounds__(kThreads) row_stats_kernel(
+    const void* __restrict__ target, const int32_t* __restrict__ path, int M,
+    const void* __restrict__ drafter, int B, int P, int V, float c,
+    RowStat* __restrict__ stats) {
+  constexpr int kV = Elem<DT>::kVec;
+  constexpr int kChunk = kThreads * kUnroll * kV;
+  __shared__ float red_m[kWarps];
+  __shared__ int red_a[kWarps];
+  __shared__ float red_s[kWarps];
+
+  const int64_t r = blockIdx.x;
+  const int64_t BP = int64_t(B) * P;
+  bool bad_path = false;
+  const void* row = r < BP ? target_row<DT>(target, path, M, P, r, V, &bad_path)
+                           : row_ptr<DT>(drafter, r - BP, V);
+
+  // pass 1: NaN-propagating max and the first index holding it
+  float m = -INFINITY;
+  int arg = INT_MAX;
+  for (int64_t v0 = 0; v0 < V; v0 += kChunk) {
+    float x[kUnroll * kV];
+    load_slots<DT, VEC>(row, v0, V, x);
+    // a thread visits its slots in increasing v, so a strict '>' keeps the
+    // first index of the maximum; a NaN replaces m and then stays
+#pragma unroll
+    for (int s = 0; s < kUnroll * kV; ++s) {
+      int64_t v = slot_pos<DT, VEC>(v0, s, threadIdx.x);
+      if (v < V && (x[s] > m || x[s] != x[s])) {
+        m = x[s];
+        arg = int(v);
+      }
+    }
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  float wm = warp_max_nan(m);
+  int wa = warp_min_int((m == wm) ? arg : INT_MAX);
+  if (l == 0) { red_m[w] = wm; red_a[w] = wa; }
+  __syncthreads();
+  float rm = red_m[0];
+  for (int j = 1; j < kWarps; ++j) rm = max_nan(rm, red_m[j]);
+  int ra = INT_MAX;
+  for (int j = 0; j < kWarps; ++j)
+    if (red_m[j] == rm && red_a[j] < ra) ra = red_a[j];
+  const bool valid = isfinite(rm) && !bad_path;
+
+  float inv_s = 0.f, mc = rm * c;
+  if (!GREEDY && valid) {
+    // pass 2: S = sum_v 2^{z_v c - m c}
+    float acc = 0.f;
+    for (int64_t v0 = 0; v0 < V; v0 += kChunk) {
+      float x[kUnroll * kV];
+      load_slots<DT, VEC>(row, v0, V, x);
+#pragma unroll
+      for (int s = 0; s < kUnroll * kV; ++s) acc += ex2(fmaf(x[s], c, -mc));
+    }
+    inv_s = 1.f / block_sum(acc, red_s);
+  }
+  if (threadIdx.x == 0) {
+    RowStat st;
+    st.m = rm;
+    st.mc = mc;
+    st.inv_s = inv_s;
+    st.argmax = valid ? ra : (bad_path ? -2 : -1);
+    stats[r] = st;
+  }
+}
+
+template <int DT, bool VEC>
+__global__ void __launch_bounds__(kThreads) overlap_kernel(
+    const void* __restrict__ target, const int32_t* __restrict__ path, int M,
+    const void* __restrict__ drafter, int N, int B, int P, int V, float c,
+    const RowStat* __restrict__ stats, float* __restrict__ partial, int nchunk) {
+  constexpr int kV = Elem<DT>::kVec;
+  constexpr int kS = kUnroll * kV;
+  constexpr int kChunk = kThreads * kS;
+  extern __shared__ float red[];  // [kWarps][N]
+
+  const int64_t tile = blockIdx.x;
+  const int j = blockIdx.y;
+  const int64_t b = tile / P, k = tile % P;
+  const int64_t BP = int64_t(B) * P;
+  const int64_t v0 = int64_t(j) * kChunk;
+  bool bad_path = false;
+  const void* trow = target_row<DT>(target, path, M, P, tile, V, &bad_path);
+  const RowStat st = stats[tile];
+
+  float p[kS];
+  load_slots<DT, VEC>(trow, v0, V, p);
+#pragma unroll
+  for (int s = 0; s < kS; ++s) p[s] = ex2(fmaf(p[s], c, -st.mc)) * st.inv_s;
+
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  for (int i = 0; i < N; ++i) {
+    const int64_t drow = (int64_t(i) * B + b) * P + k;
+    const RowStat sd = stats[BP + drow];
+    float q[kS];
+    load_slots<DT, VEC>(row_ptr<DT>(drafter, drow, V), v0, V, q);
+    float acc = 0.f;
+#pragma unroll
+    for (int s = 0; s < kS; ++s) acc += fminf(p[s], ex2(fmaf(q[s], c, -sd.mc)) * sd.inv_s);
+    acc = warp_sum(acc);
+    if (l == 0) red[w * N + i] = acc;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < N; i += kThreads) {
+    float s = 0.f;
+    for (int ww = 0; ww < kWarps; ++ww) s += red[ww * N + i];
+    partial[(tile * nchunk + j) * N + i] = s;
+  }
+}
+
+__global__ void finalize_kernel(const RowStat* __restrict__ stats,
+                                const float* __restrict__ partial, int nchunk, int N,
+                                int B, int P, int greedy, float* __restrict__ alpha,
+                                float* __restrict__ e_len, int* dev_status) {
+  const int64_t idx = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= int64_t(N) * B) return;
+  const int64_t i = idx / B, b = idx % B;
+  const int64_t BP = int64_t(B) * P;
+  float e = 1.f, prod = 1.f;
+  int err = HS_OK;
+  for (int k = 0; k < P; ++k) {
+    const int64_t tile = b * P + k;
+    const int64_t drow = (i * B + b) * P + k;
+    const RowStat st = stats[tile], sd = stats[BP + drow];
+    float a;
+    if (st.argmax < 0 || sd.argmax < 0) {
+      a = __int_as_float(0x7fc00000);  // NaN
+      if (err == HS_OK) err = (st.argmax == -2) ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE;
+    } else if (greedy) {
+      a = (st.argmax == sd.argmax) ? 1.f : 0.f;
+    } else {
+      a = 0.f;
+      const float* pp = partial + tile * int64_t(nchunk) * N + i;
+      for (int j = 0; j < nchunk; ++j) a += pp[int64_t(j) * N];
+    }
+    alpha[drow] = a;
+    if (k < P - 1) {
+      prod *= a;
+      e += prod;
+    }
+  }
+  if (e_len) e_len[idx] = e;
+  if (err != HS_OK) report(dev_status, err);
+}
+
+int elem_bytes(int dtype) { return dtype == HS_FP32 ? 4 : 2; }
+int vec_elems(int dtype) { return dtype == HS_FP32 ? 4 : 8; }
+int64_t chunk_elems(int dtype) { return int64_t(kThreads) * kUnroll * vec_elems(dtype); }
+
+struct Layout {
+  int nchunk;
+  size_t stats_off, partial_off, total;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool sizes_ok(int N, int B, int P, int V) {
+  if (N < 1 || B < 1 || P < 1 || V < 1) return false;
+  const int64_t rows = int64_t(B) * P * (int64_t(N) + 1);
+  if (rows >= (int64_t(1) << 31)) return false;  // one CTA per row
+  if (int64_t(N) * B >= (int64_t(1) << 31)) return false;
+  return double(rows) * double(V) < 4.6e18;
+}
+
+Layout layout(int N, int B, int P, int V, int dtype, int greedy) {
+  Layout L;
+  const int64_t rows = int64_t(B) * P * (int64_t(N) + 1);
+  L.nchunk = int((V + chunk_elems(dtype) - 1) / chunk_elems(dtype));
+  L.stats_off = 0;
+  L.partial_off = align256(size_t(rows) * sizeof(RowStat));
+  const size_t partial = greedy ? 0 : size_t(B) * P * L.nchunk * size_t(N) * sizeof(float);
+  L.total = L.partial_off + align256(partial);
+  return L;
+}
+
+template <int DT, bool VEC>
+hs_status launch_two_pass(const void* target, const int32_t* path, int M, const void* drafter,
+                          int N, int B, int P, int V, float c, int greedy, float* alpha,
+                          float* e_len, void* ws, const Layout& L, int* dev_status,
+                          cudaStream_t stream) {
+  RowStat* stats = reinterpret_cast<RowStat*>(static_cast<char*>(ws) + L.stats_off);
+  float* partial = reinterpret_cast<float*>(static_cast<char*>(ws) + L.partial_off);
+  const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
+  if (greedy)
+    row_stats_kernel<DT, VEC, true><<<rows, kThreads, 0, stream>>>(target, path, M, drafter, B,
+                                                                   P, V, c, stats);
+  else
+    row_stats_kernel<DT, VEC, false><<<rows, kThreads, 0, stream>>>(target, path, M, drafter,
+                                                                    B, P, V, c, stats);
+  if (!greedy) {
+    const size_t smem = size_t(kWarps) * N * sizeof(float);
+    dim3 grid(unsigned(int64_t(B) * P), unsigned(L.nchunk));
+    overlap_kernel<DT, VEC><<<grid, kThreads, smem, stream>>>(target, path, M, drafter, N, B, P,
+                                                             V, c, stats, partial, L.nchunk);
+  }
+  const int64_t nb = int64_t(N) * B;
+  finalize_kernel<<<unsigned((nb + 127) / 128), 128, 0, stream>>>(
+      stats, partial, L.nchunk, N, B, P, greedy, alpha, e_len, dev_status);
+  return cudaGetLastError() == cudaSuccess ? HS_OK : HS_ERR_CUDA;
+}
+
+template <int DT>
+hs_status dispatch_vec(bool vec, const void* target, const int32_t* path, int M,
+                       const void* drafter, int N, int B, int P, int V, float c, int greedy,
+                       float* alpha, float* e_len, void* ws, const Layout& L, int* dev_status,
+                       cudaStream_t stream) {
+  if (vec)
+    return launch_two_pass<DT, true>(target, path, M, drafter, N, B, P, V, c, greedy, alpha,
+                                     e_len, ws, L, dev_status, stream);
+  return launch_two_pass<DT, false>(target, path, M, drafter, N, B, P, V, c, greedy, alpha,
+                                    e_len, ws, L, dev_status, stream);
+}
+
+constexpr int kMaxFeedbackN = 1024;  // overlap_kernel keeps [8][N] partials in shared memory
+
+hs_status feedback_common(const void* target, const int32_t* path, int M, const void* drafter,
+                          int dtype, int N, int B, int P, int V, float temperature, int greedy,
+                          float* alpha, float* e_len, void* ws, size_t ws_bytes,
+                          int* dev_status, void* stream) {
+  if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return HS_ERR_INVALID_ARG;
+  if (!sizes_ok(N, B, P, V)) return HS_ERR_INVALID_ARG;
+  if (N > kMaxFeedbackN) return HS_ERR_UNSUPPORTED;
+  if (!target || !drafter || !alpha) return HS_ERR_INVALID_ARG;
+  if (!greedy && !(isfinite(temperature) && temperature > 0.f)) return HS_ERR_INVALID_ARG;
+  const int esz = elem_bytes(dtype);
+  if (reinterpret_cast<uintptr_t>(target) % esz || reinterpret_cast<uintptr_t>(drafter) % esz ||
+      reinterpret_cast<uintptr_t>(alpha) % 4 || reinterpret_cast<uintptr_t>(e_len) % 4 ||
+      reinterpret_cast<uintptr_t>(dev_status) % 4)
+    return HS_ERR_MISALIGNED;
+  const Layout L = layout(N, B, P, V, dtype, greedy);
+  if (L.total > 0) {
+    if (!ws || ws_bytes < L.total) return HS_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(ws) % 256) return HS_ERR_MISALIGNED;
+  }
+  const bool vec = (int64_t(V) * esz) % 16 == 0 && reinterpret_cast<uintptr_t>(target) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(drafter) % 16 == 0;
+  const float c = greedy ? 0.f : kLog2e / temperature;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (dtype) {
+    case HS_BF16:
+      return dispatch_vec<HS_BF16>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
+                                   e_len, ws, L, dev_status, s);
+    case HS_FP16:
+      return dispatch_vec<HS_FP16>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
+                                   e_len, ws, L, dev_status, s);
+    default:
+      return dispatch_vec<HS_FP32>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
+                                   e_len, ws, L, dev_status, s);
+  }
+}
+
+}  // namespace
+}  // namespace hs
+
+extern "C" size_t hs_feedback_workspace_size(int N, int B, int P, int V, int dtype, int greedy) {
+  if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return 0;
+  if (!hs::sizes_ok(N, B, P, V)) return 0;
+  return hs::layout(N, B, P, V, dtype, greedy).total;
+}
+
+extern "C" int hs_feedback_kernel_count(int N, int B, int P, int V, int dtype, int greedy) {
+  if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return 0;
+  if (!hs::sizes_ok(N, B, P, V)) return 0;
+  return greedy ? 2 : 3;
+}
+
+extern "C" hs_status hs_feedback(const void* target, const void* drafter, int dtype, int N, int B,
+                                 int P, int V, float temperature, int greedy, float* alpha,
+                                 float* e_len, void* workspace, size_t workspace_bytes,
+                                 int* dev_status, void* stream) {
+  return hs::feedback_common(target, nullptr, 0, drafter, dtype, N, B, P, V, temperature, greedy,
+                             alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" hs_status hs_feedback_path(const void* tree_target, const int32_t* path_idx, int M,
+                                      const void* drafter, int dtype, int N, int B, int P, int V,
+                                      float temperature, int greedy, float* alpha, float* e_len,
+                                      void* workspace, size_t workspace_bytes, int* dev_status,
+                                      void* stream) {
+  if (!path_idx || M < 1) return HS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(path_idx) % 4) return HS_ERR_MISALIGNED;
+  if (double(B) * double(M) * double(V) >= 4.6e18) return HS_ERR_INVALID_ARG;
+  return hs::feedback_common(tree_target, path_idx, M, drafter, dtype, N, B, P, V, temperature,
+                             greedy, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}

@@ -1,0 +1,228 @@
+"""hs_feedback / hs_feedback_path against the fp64 oracle, through the C ABI.
+
+Reduced cases keep the paper-shaped vocabularies (V = 128256 / 151936, so
+every row spans many vocab chunks and ends in a ragged one) with fewer
+drafters, queries or positions, and are compared element by element.
+Full-size cases run the benchmark's exact sizes and compare sampled outputs
+(oracle alpha one row pair at a time) and, for greedy mode, everything.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2510_20064_gb300 as hf
+from paper_2510_20064_gb300 import synth
+from parity_util import (RTOL_ALPHA, assert_rel, oracle_alpha_rows, oracle_feedback, to_np)
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+W = synth.WORKLOADS
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    hf.lib()
+    assert torch.cuda.is_available()
+
+
+def run(d, T, greedy, **kw):
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    if "path" in d:
+        a, e = hf.hs_feedback_path(d["target"], d["path"], d["drafter"], T, greedy,
+                                   dev_status=status, **kw)
+    else:
+        a, e = hf.hs_feedback(d["target"], d["drafter"], T, greedy, dev_status=status, **kw)
+    torch.cuda.synchronize()
+    return to_np(a), to_np(e), int(status.item())
+
+
+def compare_full(d, T, greedy):
+    a, e, st = run(d, T, greedy)
+    ra, re, rst = oracle_feedback(d, T, greedy)
+    assert st == hf.HS_OK and rst == 0
+    if greedy:
+        assert np.array_equal(a, ra), "greedy alpha must be bit-exact"
+        assert np.array_equal(e, re), "greedy e_len must be bit-exact"
+    else:
+        assert_rel(a, ra, RTOL_ALPHA, "alpha")
+        assert_rel(e, re, RTOL_ALPHA, "e_len")
+    return a, e
+
+
+REDUCED = [
+    ("tiny_chain", {}, (False, True)),
+    ("qwen3_8b_chain", dict(B=2), (False, True)),
+    ("llama3_batch", dict(B=3, N=8), (False, True)),
+    ("tree_path", dict(B=2), (False, True)),
+    ("long_session", dict(B=2), (False, True)),
+]
+
+
+@pytest.mark.parametrize("name,sizes,modes", REDUCED, ids=[r[0] for r in REDUCED])
+def test_reduced_workloads(name, sizes, modes):
+    w = W[name]
+    d = synth.make_inputs(w, device=DEV, **sizes)
+    for greedy in modes:
+        compare_full(d, w.temperature, greedy)
+
+
+@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 1000, 8191, 8193, 20001, 151937])
+@pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
+def test_ragged_vocab(V, dtype):
+    w = synth.Workload("ragged", N=3, B=2, P=3, V=V, dtype=dtype, temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=100 + V)
+    compare_full(d, 0.9, False)
+    compare_full(d, 0.9, True)
+
+
+@pytest.mark.parametrize("T", [0.05, 0.3, 1.0, 5.0])
+def test_temperatures(T):
+    w = W["llama3_batch"]
+    d = synth.make_inputs(w, device=DEV, B=1, N=4, P=3)
+    compare_full(d, T, False)
+
+
+def test_identical_and_disjoint_rows():
+    g = torch.Generator(device=DEV).manual_seed(5)
+    B, P, V, N = 2, 4, 40000, 3
+    tgt = torch.randn(B, P, V, generator=g, device=DEV).to(torch.bfloat16)
+    drf = tgt[None].repeat(N, 1, 1, 1).contiguous()
+    a, e, st = run({"target": tgt, "drafter": drf}, 0.8, False)
+    assert st == 0 and np.all(np.abs(a - 1) < 1e-5) and np.all(np.abs(e - P) < 1e-4)
+    a, e, st = run({"target": tgt, "drafter": drf}, 0.8, True)
+    assert np.all(a == 1) and np.all(e == P)
+    neg = torch.tensor(float("-inf"), device=DEV, dtype=torch.bfloat16)
+    even = torch.arange(V, device=DEV) % 2 == 0
+    t2 = torch.where(even, tgt, neg).contiguous()
+    d2 = torch.where(~even, drf, neg).contiguous()
+    a, e, st = run({"target": t2, "drafter": d2}, 0.8, False)
+    assert st == 0 and np.all(a == 0.0) and np.all(e == 1.0)
+
+
+def test_nonfinite_rows_flagged():
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=3, P=3, V=5000)
+    d["drafter"][1, 0, 2, 17] = float("nan")
+    d["drafter"][2, 1, 0, :] = float("-inf")
+    d["target"][1, 1, 4999] = float("inf")
+    for greedy in (False, True):
+        a, e, st = run(d, 1.0, greedy)
+        assert st == hf.HS_ERR_NONFINITE
+        ra, re, rst = oracle_feedback(d, 1.0, greedy)
+        assert rst == hf.HS_ERR_NONFINITE
+        assert np.isnan(a[1, 0, 2]) and np.isnan(a[2, 1, 0]) and np.all(np.isnan(a[:, 1, 1]))
+        if greedy:
+            assert np.array_equal(np.isnan(a), np.isnan(ra))
+            ok = ~np.isnan(ra)
+            assert np.array_equal(a[ok], ra[ok])
+        else:
+            assert_rel(a, ra, RTOL_ALPHA, "alpha with NaN rows")
+            assert_rel(e, re, RTOL_ALPHA, "e_len with NaN rows")
+
+
+def test_masked_vocabulary():
+    """-inf entries are legal: masked tokens carry probability 0."""
+    w = W["llama3_batch"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=2, P=3, V=10000)
+    mask = torch.rand(d["target"].shape[-1], device=DEV) < 0.3
+    d["target"][..., mask] = float("-inf")
+    d["drafter"][..., mask.roll(7)] = float("-inf")
+    compare_full(d, 1.0, False)
+    compare_full(d, 1.0, True)
+
+
+def test_degenerate_sizes():
+    w = W["qwen3_8b_chain"]
+    for N, B, P, V in ((1, 1, 1, 1), (1, 1, 1, 5), (1, 3, 1, 300), (5, 1, 2, 1)):
+        d = synth.make_inputs(w, device=DEV, N=N, B=B, P=P, V=V)
+        a, e = compare_full(d, 0.7, False)
+        if P == 1:
+            assert np.all(e == 1.0)
+        if V == 1:
+            assert np.allclose(a, 1.0)
+        compare_full(d, 0.7, True)
+
+
+def test_greedy_ties_lowest_index():
+    B, P, V = 1, 2, 64
+    tgt = torch.zeros(B, P, V, device=DEV, dtype=torch.bfloat16)
+    drf = torch.zeros(2, B, P, V, device=DEV, dtype=torch.bfloat16)
+    tgt[0, 0, [5, 9]] = 3.0       # target argmax = 5 (first of the tie)
+    drf[0, 0, 0, [9, 5]] = 3.0    # same tie: argmax 5 -> accepted
+    drf[1, 0, 0, 9] = 3.0         # argmax 9 -> rejected
+    tgt[0, 1, 60] = -0.0          # all zeros: first index 0 wins
+    a, _, _ = run({"target": tgt, "drafter": drf}, 1.0, True)
+    assert a[0, 0, 0] == 1.0 and a[1, 0, 0] == 0.0 and a[0, 0, 1] == 1.0 and a[1, 0, 1] == 1.0
+
+
+def test_unaligned_views_take_the_scalar_path():
+    """Logit tensors starting one element past a 16-byte boundary."""
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=2, P=3, V=4096)
+    buf_t = torch.empty(d["target"].numel() + 1, dtype=torch.bfloat16, device=DEV)
+    buf_d = torch.empty(d["drafter"].numel() + 1, dtype=torch.bfloat16, device=DEV)
+    t = buf_t[1:].view(d["target"].shape)
+    dr = buf_d[1:].view(d["drafter"].shape)
+    t.copy_(d["target"])
+    dr.copy_(d["drafter"])
+    assert t.data_ptr() % 16 != 0
+    compare_full({"target": t, "drafter": dr}, 0.7, False)
+
+
+def test_path_index_out_of_range():
+    w = W["tree_path"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=2)
+    d["path"][1, 2] = w.M  # one past the last node
+    a, e, st = run(d, 1.0, False)
+    assert st == hf.HS_ERR_INVALID_ARG
+    assert np.all(np.isnan(a[:, 1, 2])) and not np.any(np.isnan(a[:, 0, :]))
+
+
+def test_workspace_and_outputs_reused():
+    """Two calls in a row on the same buffers give identical results."""
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=4, P=3)
+    a1, e1, _ = run(d, 0.7, False)
+    a2, e2, _ = run(d, 0.7, False)
+    assert np.array_equal(a1, a2) and np.array_equal(e1, e2)
+
+
+# ---- full benchmark sizes ---------------------------------------------------
+
+FULL = ["qwen3_8b_chain", "llama3_batch", "tree_path", "long_session"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled(name):
+    w = W[name]
+    d = synth.make_inputs(w, device=DEV)
+    rng = np.random.default_rng(sum(name.encode()))
+    for greedy in sorted(set(w.greedy) | {False}):
+        a, e, st = run(d, w.temperature, greedy)
+        assert st == 0
+        samples = [(int(rng.integers(w.N)), int(rng.integers(w.B)), int(rng.integers(w.P)))
+                   for _ in range(12)]
+        samples.append((w.N - 1, w.B - 1, w.P - 1))
+        ref = oracle_alpha_rows(d, samples, w.temperature, greedy)
+        got = np.array([a[s] for s in samples])
+        if greedy:
+            assert np.array_equal(got, ref)
+        else:
+            assert_rel(got, ref, RTOL_ALPHA, f"{name} sampled alpha")
+        # e_len of two whole (i, b) columns
+        for i, b in ((0, 0), (w.N - 1, w.B - 1)):
+            col = oracle_alpha_rows(d, [(i, b, k) for k in range(w.P)], w.temperature, greedy)
+            ref_e = 1.0 + np.cumprod(col[:-1]).sum()
+            assert_rel(np.array([e[i, b]]), np.array([ref_e]), RTOL_ALPHA, f"{name} e_len")
+        # properties that hold at any size
+        ok = ~np.isnan(a)
+        assert ok.all()
+        assert np.all(a >= 0) and np.all(a <= 1 + 1e-5)
+        assert np.all(e >= 1 - 1e-6) and np.all(e <= w.P + 1e-4)
+
+
+def test_full_size_greedy_everything():
+    w = W["llama3_batch"]
+    d = synth.make_inputs(w, device=DEV)
+    compare_full(d, w.temperature, True)
