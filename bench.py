@@ -54,39 +54,6 @@ def parse_args():
     return ap.parse_args()
 
 
-# ---- distributed plumbing ---------------------------------------------------
-
-def dist_info():
-    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
-            int(os.environ.get("LOCAL_RANK", 0)))
-
-
-def dist_init(world, backend):
-    if world > 1:
-        import torch.distributed as dist
-        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
-        dist.init_process_group(backend=backend)
-
-
-def barrier(world, device=None):
-    if world > 1:
-        import torch.distributed as dist
-        if device is not None:
-            dist.barrier(device_ids=[device.index])
-        else:
-            dist.barrier()
-
-
-def max_over_ranks(x: float, world: int, device=None) -> float:
-    if world == 1:
-        return x
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
-
-
 # ---- clocks during the timed region -----------------------------------------
 
 class ClockSampler:
@@ -228,13 +195,14 @@ def run_ours(args):
     import torch
 
     import paper_2510_20064_gb300 as hf
+    from paper_2510_20064_gb300 import dist as hdist
     from paper_2510_20064_gb300 import synth
 
-    rank, world, local = dist_info()
+    rank, world, local = hdist.rank_info()
     assert torch.cuda.is_available(), "bench.py needs a GPU"
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    dist_init(world, "nccl")
+    hdist.init("nccl", world)
     hf.lib()
 
     w = synth.WORKLOADS[args.workload]
@@ -244,7 +212,7 @@ def run_ours(args):
     props = torch.cuda.get_device_properties(dev)
     l2 = getattr(props, "L2_cache_size", 0) or 129 * 2**20
     n_sets = max(2, math.ceil(2 * l2 / w.bytes_per_call))
-    sets = [synth.make_inputs(w, rnd=s, device=dev, seed=w.seed_base + 100000 * rank + s)
+    sets = [synth.make_inputs(w, rnd=s, device=dev, seed=hdist.rank_seed(w.seed_base, rank) + s)
             for s in range(n_sets)]
 
     stream = torch.cuda.Stream(device=dev)
@@ -290,21 +258,23 @@ def run_ours(args):
         full, rem = divmod(steps, per_graph)
         g_full = capture(fn, per_graph) if full else None
         g_rem = capture(fn, rem) if rem else None
-        for _ in range(2):  # graph warm-up
-            (g_full or g_rem).replay()
+        with torch.cuda.stream(stream):
+            for _ in range(2):  # graph warm-up
+                (g_full or g_rem).replay()
         stream.synchronize()
-        barrier(world, dev)
+        hdist.barrier(world, dev)
         torch.cuda.synchronize(dev)
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        for _ in range(full):
-            g_full.replay()
-        if rem:
-            g_rem.replay()
-        t1.record(stream)
+        with torch.cuda.stream(stream):  # replay() launches on the current stream
+            t0.record(stream)
+            for _ in range(full):
+                g_full.replay()
+            if rem:
+                g_rem.replay()
+            t1.record(stream)
         torch.cuda.synchronize(dev)
-        barrier(world, dev)
+        hdist.barrier(world, dev)
         return t0.elapsed_time(t1) / 1e3
 
     clocks = ClockSampler(gpu_uuid(dev))
@@ -324,7 +294,7 @@ def run_ours(args):
     d2h = out_w.numel() * 4 + out_s.numel() * 4
     e2e_steps = max(1, min(args.steps, args.e2e_steps))
     with torch.cuda.stream(stream):
-        barrier(world, dev)
+        hdist.barrier(world, dev)
         torch.cuda.synchronize(dev)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
@@ -341,9 +311,9 @@ def run_ours(args):
         torch.cuda.synchronize(dev)
     t_e2e = e0.elapsed_time(e1) / 1e3
 
-    t_step = max_over_ranks(t_step, world, dev)
-    t_fb = max_over_ranks(t_fb, world, dev)
-    t_e2e = max_over_ranks(t_e2e, world, dev)
+    t_step = hdist.max_over_ranks(t_step, world, dev)
+    t_fb = hdist.max_over_ranks(t_fb, world, dev)
+    t_e2e = hdist.max_over_ranks(t_e2e, world, dev)
     evals_step = w.evals
     value = world * args.steps * evals_step / t_step
     peak, peak_src = measured_hbm_peak()
@@ -381,14 +351,13 @@ def run_ours(args):
             "clocks": clk,
         }
         print(json.dumps(line), flush=True)
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+    hdist.finalize(world)
 
 
 def run_reference(args):
     """The fp64 CPU oracle on the host cores, same metric and config."""
-    rank, world, _ = dist_info()
+    from paper_2510_20064_gb300 import dist as hdist
+    rank, world, _ = hdist.rank_info()
     if rank != 0:
         return
     import oracle

@@ -102,6 +102,68 @@ __device__ __forceinline__ int warp_min_int(int v) {
   return v;
 }
 
+// ---- vocabulary chunks ------------------------------------------------------
+// A chunk of THREADS * UNROLL * kVec consecutive logits of one row: with VEC,
+// slot s of thread t is element v0 + ((s / kVec) * THREADS + t) * kVec +
+// s % kVec (16-byte loads, coalesced across the block); without VEC (rows
+// not 16-byte aligned) it is v0 + s * THREADS + t.  A thread's slots visit
+// increasing v either way.
+
+template <int DT, bool VEC, int THREADS>
+__device__ __forceinline__ int64_t slot_pos(int64_t v0, int s, int t) {
+  constexpr int kV = Elem<DT>::kVec;
+  if (VEC) return v0 + (int64_t((s / kV) * THREADS + t)) * kV + (s % kV);
+  return v0 + int64_t(s) * THREADS + t;
+}
+
+// Load one chunk of a row into x[] (-inf past the end of the row).
+template <int DT, bool VEC, int THREADS, int UNROLL>
+__device__ __forceinline__ void load_chunk(const void* row, int64_t v0, int V,
+                                           float (&x)[UNROLL * Elem<DT>::kVec]) {
+  constexpr int kV = Elem<DT>::kVec;
+  const int t = threadIdx.x;
+#pragma unroll
+  for (int u = 0; u < UNROLL; ++u) {
+    if (VEC) {
+      const int64_t v = v0 + int64_t(u * THREADS + t) * kV;
+      float tmp[kV];
+      if (v < V) {
+        Elem<DT>::vec(row, v, tmp);
+      } else {
+#pragma unroll
+        for (int e = 0; e < kV; ++e) tmp[e] = -INFINITY;
+      }
+#pragma unroll
+      for (int e = 0; e < kV; ++e) x[u * kV + e] = tmp[e];
+    } else {
+#pragma unroll
+      for (int e = 0; e < kV; ++e) {
+        const int64_t v = slot_pos<DT, false, THREADS>(v0, u * kV + e, t);
+        x[u * kV + e] = v < V ? Elem<DT>::one(row, v) : -INFINITY;
+      }
+    }
+  }
+}
+
+template <int DT>
+__device__ __forceinline__ const void* row_ptr(const void* base, int64_t row, int V) {
+  return static_cast<const char*>(base) + row * int64_t(V) * Elem<DT>::kBytes;
+}
+
+// Target row of tile (b,k) = b*P + k: a chain row, or the path node of a
+// draft tree (an out-of-range node reads node 0 and sets *bad_path).
+template <int DT>
+__device__ __forceinline__ const void* target_row(const void* target, const int32_t* path,
+                                                  int M, int P, int64_t tile, int V,
+                                                  bool* bad_path) {
+  if (!path) return row_ptr<DT>(target, tile, V);
+  const int64_t b = tile / P;
+  int node = path[tile];
+  *bad_path = node < 0 || node >= M;
+  if (*bad_path) node = 0;
+  return row_ptr<DT>(target, b * M + node, V);
+}
+
 // Record a data error for the caller without overwriting an earlier one.
 __device__ __forceinline__ void report(int* dev_status, int code) {
   if (dev_status) atomicCAS(dev_status, HS_OK, code);

@@ -1,21 +1,25 @@
-// hs_feedback.cu -- panoramic feedback: alpha[N,B,P] and e_len[N,B].
+// hs_feedback.cu -- hs_feedback / hs_feedback_path: argument checks and the
+// choice of kernels, plus the two-pass stochastic kernels.
 //
-// Two-pass path, used for greedy mode (where it reads every logit once) and
-// for stochastic rows that the fused cluster kernel does not take:
-//   row_stats_kernel  one CTA per logit row: max, first argmax and
+// Stochastic rows go to the single-read cluster kernel (hs_fused.cu) when it
+// takes them (bf16/fp16, V % 8 == 0, 16-byte-aligned logits, N <= 32, V up to
+// 153600); greedy rows go to the argmax kernels (hs_greedy.cu).  Everything
+// else takes the two-pass path below, which reads each logit twice:
+//   row_stats_kernel  one CTA per logit row: max and
 //                     S = sum_v 2^{(z_v - m) log2e / T}   (Thm 1's softmax)
 //   overlap_kernel    one CTA per ((b,k) tile, vocab chunk): p_v built once
 //                     and reused for all N drafters, sum_v min(p_v, q_{i,v})
 //                     (Thm 1), one partial sum per chunk
 //   finalize_kernel   one thread per (i,b): alpha over the P positions from
-//                     the partials (fixed order) or from the argmaxes
-//                     (greedy, Thm 2 with L = 1), then e_len (Thm 3).
+//                     the partials in a fixed order, then e_len (Thm 3).
 #include <math.h>
 #include <stdint.h>
 
 #include <climits>
 
 #include "hs_common.cuh"
+#include "hs_fused.h"
+#include "hs_greedy.h"
 
 namespace hs {
 
@@ -33,59 +37,10 @@ struct RowStat {
   int argmax;   // first index of m
 };
 
-template <int DT>
-__device__ __forceinline__ const void* row_ptr(const void* base, int64_t row, int V) {
-  return static_cast<const char*>(base) + row * int64_t(V) * Elem<DT>::kBytes;
-}
-
-// Target row of tile (b,k): a chain row, or the path node of a tree.
-template <int DT>
-__device__ __forceinline__ const void* target_row(const void* target, const int32_t* path,
-                                                  int M, int P, int64_t tile, int V,
-                                                  bool* bad_path) {
-  if (!path) return row_ptr<DT>(target, tile, V);
-  int64_t b = tile / P;
-  int node = path[tile];
-  *bad_path = node < 0 || node >= M;
-  if (*bad_path) node = 0;
-  return row_ptr<DT>(target, b * M + node, V);
-}
-
-// Element v handled by slot s of thread t in a chunk starting at v0.
-template <int DT, bool VEC>
-__device__ __forceinline__ int64_t slot_pos(int64_t v0, int s, int t) {
-  constexpr int kV = Elem<DT>::kVec;
-  if (VEC) return v0 + (int64_t((s / kV) * kThreads + t)) * kV + (s % kV);
-  return v0 + int64_t(s) * kThreads + t;
-}
-
-// Load the chunk slots of one row into x[] (-inf past the end of the row).
 template <int DT, bool VEC>
 __device__ __forceinline__ void load_slots(const void* row, int64_t v0, int V,
                                            float (&x)[kUnroll * Elem<DT>::kVec]) {
-  constexpr int kV = Elem<DT>::kVec;
-  const int t = threadIdx.x;
-#pragma unroll
-  for (int u = 0; u < kUnroll; ++u) {
-    if (VEC) {
-      int64_t v = v0 + int64_t(u * kThreads + t) * kV;
-      float tmp[kV];
-      if (v < V) {
-        Elem<DT>::vec(row, v, tmp);
-      } else {
-#pragma unroll
-        for (int e = 0; e < kV; ++e) tmp[e] = -INFINITY;
-      }
-#pragma unroll
-      for (int e = 0; e < kV; ++e) x[u * kV + e] = tmp[e];
-    } else {
-#pragma unroll
-      for (int e = 0; e < kV; ++e) {
-        int64_t v = slot_pos<DT, false>(v0, u * kV + e, t);
-        x[u * kV + e] = v < V ? Elem<DT>::one(row, v) : -INFINITY;
-      }
-    }
-  }
+  load_chunk<DT, VEC, kThreads, kUnroll>(row, v0, V, x);
 }
 
 __device__ __forceinline__ float block_sum(float v, float* red) {
@@ -100,7 +55,7 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return s;
 }
 
-template <int DT, bool VEC, bool GREEDY>
+template <int DT, bool VEC>
 __global__ void __launch_bounds__(kThreads) row_stats_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int B, int P, int V, float c,
@@ -127,7 +82,7 @@ __global__ void __launch_bounds__(kThreads) row_stats_kernel(
     // first index of the maximum; a NaN replaces m and then stays
 #pragma unroll
     for (int s = 0; s < kUnroll * kV; ++s) {
-      int64_t v = slot_pos<DT, VEC>(v0, s, threadIdx.x);
+      int64_t v = slot_pos<DT, VEC, kThreads>(v0, s, threadIdx.x);
       if (v < V && (x[s] > m || x[s] != x[s])) {
         m = x[s];
         arg = int(v);
@@ -147,7 +102,7 @@ __global__ void __launch_bounds__(kThreads) row_stats_kernel(
   const bool valid = isfinite(rm) && !bad_path;
 
   float inv_s = 0.f, mc = rm * c;
-  if (!GREEDY && valid) {
+  if (valid) {
     // pass 2: S = sum_v 2^{z_v c - m c}
     float acc = 0.f;
     for (int64_t v0 = 0; v0 < V; v0 += kChunk) {
@@ -212,13 +167,16 @@ __global__ void __launch_bounds__(kThreads) overlap_kernel(
   }
 }
 
+// One warp per (i, b): lanes sum the chunk partials of a position in a fixed
+// order (lane-strided, then a shuffle tree), so results repeat bit for bit.
 __global__ void finalize_kernel(const RowStat* __restrict__ stats,
                                 const float* __restrict__ partial, int nchunk, int N,
-                                int B, int P, int greedy, float* __restrict__ alpha,
+                                int B, int P, float* __restrict__ alpha,
                                 float* __restrict__ e_len, int* dev_status) {
-  const int64_t idx = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (idx >= int64_t(N) * B) return;
-  const int64_t i = idx / B, b = idx % B;
+  const int64_t gw = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  if (gw >= int64_t(N) * B) return;  // whole warp
+  const int l = threadIdx.x & 31;
+  const int64_t i = gw / B, b = gw % B;
   const int64_t BP = int64_t(B) * P;
   float e = 1.f, prod = 1.f;
   int err = HS_OK;
@@ -226,25 +184,24 @@ __global__ void finalize_kernel(const RowStat* __restrict__ stats,
     const int64_t tile = b * P + k;
     const int64_t drow = (i * B + b) * P + k;
     const RowStat st = stats[tile], sd = stats[BP + drow];
-    float a;
+    const float* pp = partial + tile * int64_t(nchunk) * N + i;
+    float a = 0.f;
+    for (int j = l; j < nchunk; j += 32) a += pp[int64_t(j) * N];
+    a = warp_sum(a);
     if (st.argmax < 0 || sd.argmax < 0) {
       a = __int_as_float(0x7fc00000);  // NaN
       if (err == HS_OK) err = (st.argmax == -2) ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE;
-    } else if (greedy) {
-      a = (st.argmax == sd.argmax) ? 1.f : 0.f;
-    } else {
-      a = 0.f;
-      const float* pp = partial + tile * int64_t(nchunk) * N + i;
-      for (int j = 0; j < nchunk; ++j) a += pp[int64_t(j) * N];
     }
-    alpha[drow] = a;
+    if (l == 0) alpha[drow] = a;
     if (k < P - 1) {
       prod *= a;
       e += prod;
     }
   }
-  if (e_len) e_len[idx] = e;
-  if (err != HS_OK) report(dev_status, err);
+  if (l == 0) {
+    if (e_len) e_len[gw] = e;
+    if (err != HS_OK) report(dev_status, err);
+  }
 }
 
 int elem_bytes(int dtype) { return dtype == HS_FP32 ? 4 : 2; }
@@ -260,6 +217,7 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 bool sizes_ok(int N, int B, int P, int V) {
   if (N < 1 || B < 1 || P < 1 || V < 1) return false;
+  if (V > (1 << 28)) return false;  // vocab chunks index gridDim.y (<= 65535)
   const int64_t rows = int64_t(B) * P * (int64_t(N) + 1);
   if (rows >= (int64_t(1) << 31)) return false;  // one CTA per row
   if (int64_t(N) * B >= (int64_t(1) << 31)) return false;
@@ -268,51 +226,50 @@ bool sizes_ok(int N, int B, int P, int V) {
 
 Layout layout(int N, int B, int P, int V, int dtype, int greedy) {
   Layout L;
+  if (greedy) {
+    L.nchunk = 0;
+    L.stats_off = L.partial_off = 0;
+    L.total = align256(greedy::workspace_bytes(N, B, P, V, dtype));
+    return L;
+  }
   const int64_t rows = int64_t(B) * P * (int64_t(N) + 1);
   L.nchunk = int((V + chunk_elems(dtype) - 1) / chunk_elems(dtype));
   L.stats_off = 0;
   L.partial_off = align256(size_t(rows) * sizeof(RowStat));
-  const size_t partial = greedy ? 0 : size_t(B) * P * L.nchunk * size_t(N) * sizeof(float);
+  const size_t partial = size_t(B) * P * L.nchunk * size_t(N) * sizeof(float);
   L.total = L.partial_off + align256(partial);
   return L;
 }
 
 template <int DT, bool VEC>
 hs_status launch_two_pass(const void* target, const int32_t* path, int M, const void* drafter,
-                          int N, int B, int P, int V, float c, int greedy, float* alpha,
-                          float* e_len, void* ws, const Layout& L, int* dev_status,
-                          cudaStream_t stream) {
+                          int N, int B, int P, int V, float c, float* alpha, float* e_len,
+                          void* ws, const Layout& L, int* dev_status, cudaStream_t stream) {
   RowStat* stats = reinterpret_cast<RowStat*>(static_cast<char*>(ws) + L.stats_off);
   float* partial = reinterpret_cast<float*>(static_cast<char*>(ws) + L.partial_off);
   const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
-  if (greedy)
-    row_stats_kernel<DT, VEC, true><<<rows, kThreads, 0, stream>>>(target, path, M, drafter, B,
-                                                                   P, V, c, stats);
-  else
-    row_stats_kernel<DT, VEC, false><<<rows, kThreads, 0, stream>>>(target, path, M, drafter,
-                                                                    B, P, V, c, stats);
-  if (!greedy) {
-    const size_t smem = size_t(kWarps) * N * sizeof(float);
-    dim3 grid(unsigned(int64_t(B) * P), unsigned(L.nchunk));
-    overlap_kernel<DT, VEC><<<grid, kThreads, smem, stream>>>(target, path, M, drafter, N, B, P,
-                                                             V, c, stats, partial, L.nchunk);
-  }
-  const int64_t nb = int64_t(N) * B;
-  finalize_kernel<<<unsigned((nb + 127) / 128), 128, 0, stream>>>(
-      stats, partial, L.nchunk, N, B, P, greedy, alpha, e_len, dev_status);
+  row_stats_kernel<DT, VEC><<<rows, kThreads, 0, stream>>>(target, path, M, drafter, B, P, V, c,
+                                                           stats);
+  const size_t smem = size_t(kWarps) * N * sizeof(float);
+  dim3 grid(unsigned(int64_t(B) * P), unsigned(L.nchunk));
+  overlap_kernel<DT, VEC><<<grid, kThreads, smem, stream>>>(target, path, M, drafter, N, B, P, V,
+                                                           c, stats, partial, L.nchunk);
+  const int64_t threads = int64_t(N) * B * 32;
+  finalize_kernel<<<unsigned((threads + 255) / 256), 256, 0, stream>>>(
+      stats, partial, L.nchunk, N, B, P, alpha, e_len, dev_status);
   return cudaGetLastError() == cudaSuccess ? HS_OK : HS_ERR_CUDA;
 }
 
 template <int DT>
 hs_status dispatch_vec(bool vec, const void* target, const int32_t* path, int M,
-                       const void* drafter, int N, int B, int P, int V, float c, int greedy,
-                       float* alpha, float* e_len, void* ws, const Layout& L, int* dev_status,
+                       const void* drafter, int N, int B, int P, int V, float c, float* alpha,
+                       float* e_len, void* ws, const Layout& L, int* dev_status,
                        cudaStream_t stream) {
   if (vec)
-    return launch_two_pass<DT, true>(target, path, M, drafter, N, B, P, V, c, greedy, alpha,
-                                     e_len, ws, L, dev_status, stream);
-  return launch_two_pass<DT, false>(target, path, M, drafter, N, B, P, V, c, greedy, alpha,
-                                    e_len, ws, L, dev_status, stream);
+    return launch_two_pass<DT, true>(target, path, M, drafter, N, B, P, V, c, alpha, e_len, ws,
+                                     L, dev_status, stream);
+  return launch_two_pass<DT, false>(target, path, M, drafter, N, B, P, V, c, alpha, e_len, ws, L,
+                                    dev_status, stream);
 }
 
 constexpr int kMaxFeedbackN = 1024;  // overlap_kernel keeps [8][N] partials in shared memory
@@ -340,16 +297,22 @@ hs_status feedback_common(const void* target, const int32_t* path, int M, const 
                    reinterpret_cast<uintptr_t>(drafter) % 16 == 0;
   const float c = greedy ? 0.f : kLog2e / temperature;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (greedy)
+    return greedy::launch(vec, target, path, M, drafter, dtype, N, B, P, V, alpha, e_len, ws,
+                          dev_status, s);
+  if (fused::eligible(target, drafter, dtype, N, V, greedy))
+    return fused::launch(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, dev_status,
+                         s);
   switch (dtype) {
     case HS_BF16:
-      return dispatch_vec<HS_BF16>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
-                                   e_len, ws, L, dev_status, s);
+      return dispatch_vec<HS_BF16>(vec, target, path, M, drafter, N, B, P, V, c, alpha, e_len,
+                                   ws, L, dev_status, s);
     case HS_FP16:
-      return dispatch_vec<HS_FP16>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
-                                   e_len, ws, L, dev_status, s);
+      return dispatch_vec<HS_FP16>(vec, target, path, M, drafter, N, B, P, V, c, alpha, e_len,
+                                   ws, L, dev_status, s);
     default:
-      return dispatch_vec<HS_FP32>(vec, target, path, M, drafter, N, B, P, V, c, greedy, alpha,
-                                   e_len, ws, L, dev_status, s);
+      return dispatch_vec<HS_FP32>(vec, target, path, M, drafter, N, B, P, V, c, alpha, e_len,
+                                   ws, L, dev_status, s);
   }
 }
 
@@ -365,6 +328,7 @@ extern "C" size_t hs_feedback_workspace_size(int N, int B, int P, int V, int dty
 extern "C" int hs_feedback_kernel_count(int N, int B, int P, int V, int dtype, int greedy) {
   if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return 0;
   if (!hs::sizes_ok(N, B, P, V)) return 0;
+  if (hs::fused::eligible_sizes(dtype, N, V, greedy)) return 2;  // 16-byte-aligned logits
   return greedy ? 2 : 3;
 }
 

@@ -226,3 +226,45 @@ def test_full_size_greedy_everything():
     w = W["llama3_batch"]
     d = synth.make_inputs(w, device=DEV)
     compare_full(d, w.temperature, True)
+
+
+# ---- both feedback paths ------------------------------------------------------
+# bf16/fp16 rows with V % 8 == 0, 16-byte-aligned logits and N <= 32 take the
+# single-read cluster kernel (cluster size 1, 2, 4 or 8 by V); everything
+# else takes the two-pass kernels.  These cases cross each boundary.
+
+@pytest.mark.parametrize("V", [8, 4096, 19200, 19208, 38400, 38408, 76800, 76808, 128256,
+                               151936, 153600, 153608])
+def test_cluster_sizes(V):
+    w = synth.Workload("vsweep", N=3, B=2, P=3, V=V, dtype="bf16", temperature=0.8,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=7 + V)
+    compare_full(d, 0.8, False)
+
+
+@pytest.mark.parametrize("N", [1, 31, 32, 33])
+def test_drafter_counts(N):
+    w = W["llama3_batch"]
+    d = synth.make_inputs(w, device=DEV, N=N, B=1, P=2, V=20000)
+    compare_full(d, 1.0, False)
+
+
+def test_more_tiles_than_resident_clusters():
+    """B*P = 1200 tiles: every resident cluster loops over many tiles."""
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, N=2, B=200, P=6, V=38400)
+    a, e, st = run(d, 0.7, False)
+    assert st == 0
+    rng = np.random.default_rng(3)
+    samples = [(int(rng.integers(2)), int(rng.integers(200)), int(rng.integers(6)))
+               for _ in range(40)]
+    ref = oracle_alpha_rows(d, samples, 0.7, False)
+    assert_rel(np.array([a[s] for s in samples]), ref, RTOL_ALPHA, "many-tile alpha")
+
+
+def test_fp16_full_vocab():
+    w = synth.Workload("fp16", N=4, B=2, P=3, V=151936, dtype="fp16", temperature=0.7,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=11)
+    compare_full(d, 0.7, False)
+    compare_full(d, 0.7, True)
