@@ -6,9 +6,10 @@
 // pass.  A vocabulary row (up to ~300 KB of bf16) does not fit one SM, so a
 // cluster of C CTAs takes one (b,k) tile, each CTA a V/C slice, and loops
 // persistently over tiles:
-//   * a producer warp streams the CTA's slice of every row of its tiles --
-//     the target row, then the N drafter rows -- into a 3-stage shared-memory
-//     ring with cp.async.bulk (TMA; each CTA reads its own slice, no multicast);
+//   * the CTA's slice of every row of its tiles -- the target row, then the
+//     N drafter rows -- streams into a 3-stage shared-memory ring with
+//     cp.async.bulk (TMA; each CTA reads its own slice, no multicast); a
+//     coordinator warp refills a stage as soon as every consumer has read it;
 //   * 15 consumer warps load a row from the ring into registers, form
 //     e_v = 2^{z_v c - o_w} with o_w = c * (the warp's max), c = log2e/T,
 //     and their sum (one ex2 per logit, values kept in registers);
@@ -18,10 +19,11 @@
 //     normaliser Z, and p_v or q_v = e_v 2^{o_t - O} / Z;
 //   * the target's p stays in shared memory (fp32) for the tile's N drafters;
 //     a drafter row adds sum_v min(p_v, q_v) to its per-warp partial;
-//   * at the end of a tile the producer warp sums the warps' N partials and
-//     sends them to the cluster's rank 0, whose producer warp sums them in
-//     rank order and writes alpha[:, b, k] (one tile later, off the
-//     critical path).  Consumer warps never wait for one another.
+//   * at the end of a tile the coordinator sums the warps' N partials and
+//     sends them to the cluster's rank 0, whose coordinator sums them in rank
+//     order and writes alpha[:, b, k] one tile later.  The coordinator never
+//     blocks: its waits poll, servicing ring refills meanwhile, and no
+//     consumer warp waits for another warp of its CTA.
 // Rows are software-pipelined: the pass over row g+1's logits runs while
 // row g's cluster exchange is in flight, so each thread holds two rows of
 // exponentials (eA / eB).  Every wait is bounded; on expiry the kernel
@@ -36,13 +38,17 @@ namespace hs {
 namespace fused {
 namespace {
 
-// 15 consumer warps + 1 producer warp: 16 warps put 4 on each SM
-// sub-partition, which leaves 128 registers per thread for the two rows of
-// exponentials a consumer keeps.
+// 15 consumer warps + 1 load warp: 16 warps put 4 on each SM sub-partition,
+// which leaves 128 registers per thread for the two rows of exponentials a
+// consumer thread keeps.
 constexpr int kConsumerWarps = 15;
 constexpr int kConsumers = kConsumerWarps * 32;
-constexpr int kThreads = kConsumers + 32;  // + one producer warp
+constexpr int kThreads = kConsumers + 32;
 constexpr int kStages = 3;
+// Rows ahead of the ring whose slice is prefetched into L2 (bulk prefetch,
+// no shared memory): the ring's TMA loads then hit L2, which keeps a few
+// hundred KB per SM in flight although only ~2 stages fit next to p.
+constexpr int kPrefetch = 0;
 constexpr int kXSlots = 4;  // rows whose exchange may be in flight at once
 constexpr int kASlots = 4;  // tiles whose alpha partials may be in flight
 constexpr int kMaxU = 5;    // 16-byte vectors per consumer thread and row
@@ -51,18 +57,18 @@ constexpr uint32_t kNegInfBf16x2 = 0xFF80FF80u;
 constexpr uint32_t kNegInfF16x2 = 0xFC00FC00u;
 
 struct __align__(16) Shared {
-  uint64_t full[kStages];               // ring stage loaded (TMA complete_tx)
-  uint64_t empty[kStages];              // ring stage read by every consumer warp
-  uint64_t redbar[kXSlots];             // every consumer warp posted its row pair
-  uint64_t xbar[kXSlots];               // every rank's pair of a row has arrived
-  uint64_t accbar[2];                   // every consumer warp posted a tile's partials
-  uint64_t abar[kASlots];               // every rank's tile partials arrived (rank 0)
-  float2 red[kXSlots][16];              // per-warp (offset, sum) of a row
-  float2 xch[kXSlots][kMaxC];           // per-rank (offset, sum) of a row
-  float acc[2][kMaxN][kConsumerWarps];  // per-warp alpha partials of a tile
-  uint32_t tvalid[2];                   // the tile's target row is usable
-  uint32_t dvalid[2];                   // bit i: drafter i's row is usable
-  float clacc[kASlots][kMaxC][kMaxN];   // per-rank alpha partials (rank 0)
+  uint64_t full[kStages];          // ring stage loaded (TMA complete_tx)
+  uint64_t empty[kStages];         // ring stage read by every consumer warp
+  uint64_t redbar[kXSlots];        // every consumer warp posted its row pair
+  uint64_t xbar[kXSlots];          // every rank's pair of a row arrived
+  uint64_t accbar[2];              // every consumer warp posted a tile's partials
+  uint64_t abar[kASlots];          // every rank's tile partials arrived (rank 0)
+  float2 red[kXSlots][16];                // per-warp (offset, sum) of a row
+  float2 xch[kXSlots][kMaxC];             // per-rank (offset, sum) of a row
+  float acc[2][kMaxN][kConsumerWarps];    // per-warp alpha partials of a tile
+  uint32_t tvalid[2];                     // the tile's target row is usable
+  uint32_t dvalid[2];                     // bit i: drafter i's row is usable
+  float clacc[kASlots][kMaxC][kMaxN];     // per-rank alpha partials (rank 0)
   int error;
 };
 
@@ -118,12 +124,6 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
                :: "r"(bar), "r"(bytes) : "memory");
 }
-// Arrive on a barrier in another CTA of the cluster, ordering this thread's
-// earlier shared::cluster stores before the arrival.
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];"
-               :: "r"(cluster_bar) : "memory");
-}
 // try_wait suspends the thread until the phase completes or about 1 ms has
 // passed, so a waiting warp does not spin through the issue slots.
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
@@ -140,6 +140,20 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
                "[%0], [%1], %2, [%3];"
                :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
+__device__ __forceinline__ bool mbar_probe(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n\t.reg .pred p;\n\t"
+               "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+               "selp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Arrive on a barrier in another CTA of the cluster, ordering this thread's
+// earlier shared::cluster stores before the arrival.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];"
+               :: "r"(cluster_bar) : "memory");
+}
 __device__ __forceinline__ void st_cluster_f2(uint32_t a, float x, float y) {
   asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" :: "r"(a), "f"(x), "f"(y) : "memory");
 }
@@ -153,14 +167,13 @@ __device__ __forceinline__ uint4 lds128(uint32_t a) {
   return v;
 }
 
-// Bounded wait on an mbarrier phase.  Returns false (and records a timeout
+// Bounded wait on an mbarrier phase (the slow path of wait_phase).  Returns false (and records a timeout
 // once per CTA) when the phase did not complete in time or an earlier wait
 // of this CTA already timed out.
 // The exit drain passes fast_fail = false: it must see in-flight copies land
 // even after another wait has given up.
-__device__ __noinline__ bool wait_phase(uint32_t bar, uint32_t parity, Shared& sh,
-                                        int* dev_status, bool fast_fail = true) {
-  if (mbar_test(bar, parity)) return true;
+__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, Shared& sh,
+                                       int* dev_status, bool fast_fail) {
   const long long t0 = clock64();
   while (true) {
     if (fast_fail && *reinterpret_cast<volatile int*>(&sh.error)) return false;
@@ -171,6 +184,12 @@ __device__ __noinline__ bool wait_phase(uint32_t bar, uint32_t parity, Shared& s
       return false;
     }
   }
+}
+
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, Shared& sh,
+                                           int* dev_status, bool fast_fail = true) {
+  if (mbar_test(bar, parity)) return true;
+  return wait_slow(bar, parity, sh, dev_status, fast_fail);
 }
 
 // ---- per-element helpers ----------------------------------------------------
@@ -253,14 +272,63 @@ struct Row {
   float o;        // reported offset: -inf when the warp saw no finite logit
 };
 
+// Global address of this CTA's slice of its row g: row g % (N+1) of the
+// CTA's (g / (N+1))-th tile -- the target row, then the drafter rows.
+__device__ __forceinline__ const char* row_slice(const Params& p, int g, uint32_t cid,
+                                                 uint32_t ncl, int64_t slice0) {
+  const int R = p.N + 1;
+  const int j = g / R, r = g % R;
+  const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
+  const int64_t b = tile / p.P, k = tile % p.P;
+  int64_t row;
+  const void* base;
+  if (r == 0) {
+    if (p.path) {
+      const int nd = p.path[tile];
+      row = b * p.M + ((nd < 0 || nd >= p.M) ? 0 : nd);
+    } else {
+      row = tile;
+    }
+    base = p.target;
+  } else {
+    row = (int64_t(r - 1) * p.B + b) * p.P + k;
+    base = p.drafter;
+  }
+  return static_cast<const char*>(base) + (row * p.V + slice0) * 2;
+}
+
+// Stream row g into `stage` (one thread); with kPrefetch > 0 also prefetch
+// row g + kPrefetch into L2.
+__device__ __forceinline__ void issue(const Params& p, Shared& sh, unsigned char* stage, int g,
+                                      int G, uint32_t cid, uint32_t ncl, int64_t slice0,
+                                      uint32_t bytes) {
+  const uint32_t full = saddr(&sh.full[g % kStages]);
+  if (bytes) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    mbar_arrive_tx(full, bytes);
+    bulk_load(saddr(stage), row_slice(p, g, cid, ncl, slice0), bytes, full);
+    if (kPrefetch > 0 && g + kPrefetch < G)
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                   :: "l"(row_slice(p, g + kPrefetch, cid, ncl, slice0)), "r"(bytes) : "memory");
+  } else {
+    mbar_arrive(full);
+  }
+}
+
 template <int DT, int U>
 __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Shared& sh = *reinterpret_cast<Shared*>(smem_raw);
-  const int S = p.S;
-  const size_t stage_bytes = (size_t(S) * 2 + 127) & ~size_t(127);
+  // every buffer holds SU = U * kConsumers * 8 >= S elements so that each
+  // consumer thread always handles U whole 16-byte vectors; the part past
+  // the CTA's slice is -inf in the ring and 0 in p (set once, below)
+  constexpr int SU = U * kConsumers * 8;
+  constexpr uint32_t stage_bytes = SU * 2;
   unsigned char* ring = smem_raw + ((sizeof(Shared) + 127) & ~size_t(127));
-  float* pbuf = reinterpret_cast<float*>(ring + kStages * stage_bytes);
+  // p of the tile's target, as two planes of float4 so that consecutive
+  // threads read consecutive 16 bytes: pA[vi] = p[8vi..8vi+3], pB[vi] = p[8vi+4..8vi+7]
+  float4* pA = reinterpret_cast<float4*>(ring + kStages * stage_bytes);
+  float4* pB = pA + SU / 8;
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -272,10 +340,19 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   const int my_tiles = cid < uint32_t(p.ntiles) ? int((p.ntiles - 1 - cid) / ncl) + 1 : 0;
   const int R = N + 1;        // rows per tile: the target, then the N drafters
   const int G = my_tiles * R;  // rows this CTA streams
-  const int64_t slice0 = int64_t(rank) * S;
+  const int64_t slice0 = int64_t(rank) * p.S;
   const int64_t rest = int64_t(V) - slice0;
-  const int len = rest <= 0 ? 0 : (rest < S ? int(rest) : S);
+  const int len = rest <= 0 ? 0 : (rest < p.S ? int(rest) : p.S);
+  const uint32_t bytes = uint32_t(len) * 2u;
 
+  {
+    const uint32_t neg = (DT == HS_BF16) ? kNegInfBf16x2 : kNegInfF16x2;
+    for (int e = len / 2 + tid; e < SU / 2; e += kThreads)
+      for (int s = 0; s < kStages; ++s)
+        reinterpret_cast<uint32_t*>(ring + s * stage_bytes)[e] = neg;
+    for (int vi = len / 8 + tid; vi < SU / 8; vi += kThreads)
+      pA[vi] = pB[vi] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(saddr(&sh.full[s]), 1);
@@ -293,81 +370,65 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   cluster_sync_all();
 
   if (warp == kConsumerWarps) {
-    // -------------------- producer / coordinator warp ---------------------
-    // lane 0 streams row slices into the ring; the whole warp merges the
-    // consumer warps' per-row pairs, sends them to every rank, and reduces
-    // each tile's alpha partials (rank 0 also writes alpha, one tile late).
-    const uint32_t bytes = uint32_t(len) * 2u;
-    auto issue = [&](int g) {
-      const int j = g / R, r = g % R;
-      const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
-      const int64_t b = tile / P, k = tile % P;
-      int64_t row;
-      const void* base;
-      if (r == 0) {
-        if (p.path) {
-          const int nd = p.path[tile];
-          row = b * p.M + ((nd < 0 || nd >= p.M) ? 0 : nd);
-        } else {
-          row = tile;
-        }
-        base = p.target;
-      } else {
-        row = (int64_t(r - 1) * B + b) * P + k;
-        base = p.drafter;
-      }
-      const int s = g % kStages;
-      if (g >= kStages)
-        wait_phase(saddr(&sh.empty[s]), uint32_t((g / kStages) - 1) & 1u, sh, p.dev_status);
-      const uint32_t full = saddr(&sh.full[s]);
-      if (bytes) {
-        mbar_arrive_tx(full, bytes);
-        bulk_load(saddr(ring + s * stage_bytes),
-                  static_cast<const char*>(base) + (row * V + slice0) * 2, bytes, full);
-      } else {
-        mbar_arrive(full);
+    // ---------------------------- coordinator -----------------------------
+    // Never blocks: every wait polls its barrier and, while it does, lane 0
+    // refills each ring stage as soon as all consumer warps have read it.
+    // The warp merges the consumer warps' row pairs and sends the CTA's pair
+    // to every rank, and reduces each tile's alpha partials (rank 0 also
+    // writes alpha, one tile late).
+    int issued = 0;
+    auto service = [&]() {
+      if (lane != 0) return;
+      while (issued < G &&
+             (issued < kStages ||
+              mbar_probe(saddr(&sh.empty[issued % kStages]),
+                         uint32_t((issued / kStages) - 1) & 1u))) {
+        issue(p, sh, ring + (issued % kStages) * stage_bytes, issued, G, cid, ncl, slice0, bytes);
+        ++issued;
       }
     };
-    // tile j: sum the 15 warps' partials, send them to rank 0
-    uint32_t pend_t = 0, pend_d = 0;
-    int pend_tile = -1;
-    auto finish_tile = [&](int j) {  // rank 0: alpha[:, b, k] of tile j
-      wait_phase(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u, sh, p.dev_status);
+    auto poll = [&](uint32_t bar, uint32_t parity) {
+      service();
+      const long long t0 = clock64();
+      while (!mbar_probe(bar, parity)) {
+        service();
+        if (*reinterpret_cast<volatile int*>(&sh.error)) return;
+        if (clock64() - t0 > kTimeoutCycles) {
+          *reinterpret_cast<volatile int*>(&sh.error) = 1;
+          report(p.dev_status, HS_ERR_TIMEOUT);
+          return;
+        }
+        __nanosleep(32);
+      }
+    };
+    auto finish = [&](int j) {  // rank 0: alpha[:, b, k] of tile j
+      poll(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u);
       if (lane < N) {
         const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
         const int64_t b = tile / P, k = tile % P;
         float t = 0.f;
         for (uint32_t rr = 0; rr < C; ++rr) t += sh.clacc[j % kASlots][rr][lane];
         const bool bad_path = p.path && (p.path[tile] < 0 || p.path[tile] >= p.M);
-        if (bad_path || !pend_t || !((pend_d >> lane) & 1u)) {
+        if (bad_path || !sh.tvalid[j & 1] || !((sh.dvalid[j & 1] >> lane) & 1u)) {
           t = __int_as_float(0x7fc00000);
           report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
         }
         p.alpha[(int64_t(lane) * B + b) * P + k] = t;
       }
     };
-    auto reduce_tile = [&](int j) {
-      wait_phase(saddr(&sh.accbar[j & 1]), uint32_t(j >> 1) & 1u, sh, p.dev_status);
-      const uint32_t vt = sh.tvalid[j & 1], vd = sh.dvalid[j & 1];
+    auto reduce_tile = [&](int j) {  // tile j's partials -> rank 0
+      poll(saddr(&sh.accbar[j & 1]), uint32_t(j >> 1) & 1u);
       if (lane < N) {
         float t = 0.f;
         for (int w = 0; w < kConsumerWarps; ++w) t += sh.acc[j & 1][lane][w];
         st_cluster_f(mapa(saddr(&sh.clacc[j % kASlots][rank][lane]), 0), t);
         mbar_arrive_remote(mapa(saddr(&sh.abar[j % kASlots]), 0));
       }
-      if (rank == 0) {
-        if (pend_tile >= 0) finish_tile(pend_tile);
-        pend_tile = j;
-        pend_t = vt;
-        pend_d = vd;
-      }
+      if (rank == 0 && j > 0) finish(j - 1);  // long since complete
     };
-    if (lane == 0)
-      for (int g = 0; g < min(G, kStages); ++g) issue(g);
     for (int g = 0; g < G; ++g) {
       const int x = g % kXSlots;
-      wait_phase(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
-      if (lane == 0 && g + kStages < G) issue(g + kStages);
+      poll(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u);
       float2 v = lane < kConsumerWarps ? sh.red[x][lane] : make_float2(-INFINITY, 0.f);
       float oc = v.x, sc = v.y;
       warp_merge(oc, sc);
@@ -379,23 +440,25 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       // first row of tile j+1, so reduce tile j once that row is merged
       if (g % R == 0 && g > 0) reduce_tile(g / R - 1);
     }
-    if (G > 0) reduce_tile(G / R - 1);
-    if (rank == 0 && pend_tile >= 0) finish_tile(pend_tile);
-    // drain: every copy issued has landed before the CTA may exit
+    if (G > 0) {
+      reduce_tile(my_tiles - 1);
+      if (rank == 0) finish(my_tiles - 1);
+    }
+    // every row was issued (the consumers have read them all); drain: every
+    // copy has landed before the CTA may exit
     if (lane == 0)
       for (int g = max(0, G - kStages); g < G; ++g)
         wait_phase(saddr(&sh.full[g % kStages]), uint32_t(g / kStages) & 1u, sh, p.dev_status,
                    false);
-  } else {
+  } else if (G > 0) {
     // ------------------------------ consumers -----------------------------
     const float c = p.c;
-    const uint32_t neg = (DT == HS_BF16) ? kNegInfBf16x2 : kNegInfF16x2;
     uint32_t tvalid = 0, dvalid = 0;  // target row usable; bit i: drafter i usable
     Row<DT, U> A, Bv;
 
-    // pass 1: load row g from the ring; warp max; exponentials relative to
-    // the warp's offset (kept in registers) and their sum; post the warp's
-    // (offset, sum) for the coordinator
+    // pass 1: load row g from the ring (then release the stage); warp max;
+    // exponentials relative to the warp's offset, kept in registers; post
+    // the warp's (offset, sum) for the coordinator
     auto pass1 = [&](int g, Row<DT, U>& Rw) {
       const int s = g % kStages;
       wait_phase(saddr(&sh.full[s]), uint32_t(g / kStages) & 1u, sh, p.dev_status);
@@ -403,41 +466,34 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       uint32_t w[U * 4];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int vi = u * kConsumers + tid;
-        if (vi * 8 < len) {
-          const uint4 v = lds128(stage + vi * 16);
-          w[4 * u] = v.x; w[4 * u + 1] = v.y; w[4 * u + 2] = v.z; w[4 * u + 3] = v.w;
-        } else {
-          w[4 * u] = w[4 * u + 1] = w[4 * u + 2] = w[4 * u + 3] = neg;
-        }
+        const uint4 v = lds128(stage + (u * kConsumers + tid) * 16);
+        w[4 * u] = v.x; w[4 * u + 1] = v.y; w[4 * u + 2] = v.z; w[4 * u + 3] = v.w;
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(saddr(&sh.empty[s]));
-      uint32_t mx[U * 4];  // pairwise tree: log-depth dependency chain
+      uint32_t mx[U * 2];  // pairwise tree: log-depth dependency chain
 #pragma unroll
-      for (int q = 0; q < U * 4; ++q) mx[q] = w[q];
+      for (int q = 0; q < U * 2; ++q) mx[q] = pmax<DT>(w[2 * q], w[2 * q + 1]);
 #pragma unroll
-      for (int d = 1; d < U * 4; d *= 2)
+      for (int d = 1; d < U * 2; d *= 2)
 #pragma unroll
-        for (int q = 0; q + d < U * 4; q += 2 * d) mx[q] = pmax<DT>(mx[q], mx[q + d]);
+        for (int q = 0; q + d < U * 2; q += 2 * d) mx[q] = pmax<DT>(mx[q], mx[q + d]);
       const float m = warp_max_key(max_nan(lo<DT>(mx[0]), hi<DT>(mx[0])));
       Rw.o = (m == -INFINITY) ? -INFINITY : m * c;
       Rw.o_used = (m == -INFINITY) ? 0.f : Rw.o;
       const f2_t cc = pk(c, c), off = pk(-Rw.o_used, -Rw.o_used);
-      f2_t acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
+      f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
       for (int q = 0; q < U * 4; ++q) {
         float a, b;
         upk(ffma2(pk(lo<DT>(w[q]), hi<DT>(w[q])), cc, off), a, b);
         Rw.e[q] = pk(ex2(a), ex2(b));
-        acc[q & 3] = fadd2(acc[q & 3], Rw.e[q]);
+        acc[q & 1] = fadd2(acc[q & 1], Rw.e[q]);
       }
-      float s0, s1, s2, s3, s4, s5, s6, s7;
+      float s0, s1, s2, s3;
       upk(acc[0], s0, s1);
       upk(acc[1], s2, s3);
-      upk(acc[2], s4, s5);
-      upk(acc[3], s6, s7);
-      const float sum = warp_sum(((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
+      const float sum = warp_sum((s0 + s1) + (s2 + s3));
       if (lane == 0) {
         sh.red[g % kXSlots][warp] = make_float2(Rw.o, sum);
         mbar_arrive(saddr(&sh.redbar[g % kXSlots]));
@@ -469,60 +525,52 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
 #pragma unroll
         for (int u = 0; u < U; ++u) {
           const int vi = u * kConsumers + tid;
-          if (vi * 8 < len) {
-            float q[8];
+          float q[8];
 #pragma unroll
-            for (int h = 0; h < 4; ++h) upk(fmul2(Rw.e[4 * u + h], ff), q[2 * h], q[2 * h + 1]);
-            float4* dst = reinterpret_cast<float4*>(pbuf + vi * 8);
-            dst[0] = make_float4(q[0], q[1], q[2], q[3]);
-            dst[1] = make_float4(q[4], q[5], q[6], q[7]);
-          }
+          for (int h = 0; h < 4; ++h) upk(fmul2(Rw.e[4 * u + h], ff), q[2 * h], q[2 * h + 1]);
+          pA[vi] = make_float4(q[0], q[1], q[2], q[3]);
+          pB[vi] = make_float4(q[4], q[5], q[6], q[7]);
         }
-      } else {
-        const int i = r - 1;
-        if (ok) dvalid |= 1u << i;
-        f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
+        return;
+      }
+      const int i = r - 1;
+      if (ok) dvalid |= 1u << i;
+      f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const int vi = u * kConsumers + tid;
-          if (vi * 8 < len) {
-            const float4* src = reinterpret_cast<const float4*>(pbuf + vi * 8);
-            const float4 p0 = src[0], p1 = src[1];
-            const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+      for (int u = 0; u < U; ++u) {
+        const int vi = u * kConsumers + tid;
+        const float4 p0 = pA[vi], p1 = pB[vi];
+        const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              float x, y;
-              upk(fmul2(Rw.e[4 * u + h], ff), x, y);
-              acc[h & 1] = fadd2(acc[h & 1], pk(fminf(pv[2 * h], x), fminf(pv[2 * h + 1], y)));
-            }
-          }
+        for (int h = 0; h < 4; ++h) {
+          float xx, yy;
+          upk(fmul2(Rw.e[4 * u + h], ff), xx, yy);
+          acc[h & 1] = fadd2(acc[h & 1], pk(fminf(pv[2 * h], xx), fminf(pv[2 * h + 1], yy)));
         }
-        float a0, a1, a2, a3;
-        upk(acc[0], a0, a1);
-        upk(acc[1], a2, a3);
-        const float a = warp_sum((a0 + a1) + (a2 + a3));
-        if (lane == 0) {
-          sh.acc[j & 1][i][warp] = a;
-          if (i == N - 1) {  // tile end: hand the partials to the coordinator
-            if (warp == 0) {
-              sh.tvalid[j & 1] = tvalid;
-              sh.dvalid[j & 1] = dvalid;
-            }
-            mbar_arrive(saddr(&sh.accbar[j & 1]));
+      }
+      float a0, a1, a2, a3;
+      upk(acc[0], a0, a1);
+      upk(acc[1], a2, a3);
+      const float a = warp_sum((a0 + a1) + (a2 + a3));
+      if (lane == 0) {
+        sh.acc[j & 1][i][warp] = a;
+        if (i == N - 1) {  // tile end: hand the partials to the coordinator
+          if (warp == 0) {
+            sh.tvalid[j & 1] = tvalid;
+            sh.dvalid[j & 1] = dvalid;
           }
+          mbar_arrive(saddr(&sh.accbar[j & 1]));
         }
       }
     };
 
-    if (G > 0) {
-      pass1(0, A);
-      for (int g = 0; g < G; g += 2) {
-        if (g + 1 < G) pass1(g + 1, Bv);
-        pass2(g, A);
-        if (g + 1 < G) {
-          if (g + 2 < G) pass1(g + 2, A);
-          pass2(g + 1, Bv);
-        }
+    pass1(0, A);
+    for (int g = 0; g < G; g += 2) {
+      if (g + 1 < G) pass1(g + 1, Bv);
+      pass2(g, A);
+      if (g + 1 < G) {
+        if (g + 2 < G) pass1(g + 2, A);
+        pass2(g + 1, Bv);
       }
     }
   }
@@ -533,9 +581,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
 
 // ---- host side ------------------------------------------------------------------
 
-size_t shared_bytes(int S) {
-  const size_t stage = (size_t(S) * 2 + 127) & ~size_t(127);
-  return ((sizeof(Shared) + 127) & ~size_t(127)) + kStages * stage + size_t(S) * 4;
+size_t shared_bytes(int U) {
+  const size_t SU = size_t(U) * kConsumers * 8;  // padded slice, see the kernel
+  return ((sizeof(Shared) + 127) & ~size_t(127)) + kStages * SU * 2 + SU * 4;
 }
 
 constexpr size_t kSmemLimit = 227 * 1024;
@@ -549,7 +597,7 @@ Plan plan_for(int V) {
   for (int C = 1; C <= kMaxC; C *= 2) {
     const int S = ((V + C - 1) / C + 7) / 8 * 8;
     const int U = (S + kConsumers * 8 - 1) / (kConsumers * 8);
-    if (U <= kMaxU && shared_bytes(S) <= kSmemLimit) {
+    if (U <= kMaxU && shared_bytes(U) <= kSmemLimit) {
       pl.C = C;
       pl.S = S;
       pl.U = U;
@@ -562,7 +610,7 @@ Plan plan_for(int V) {
 template <int DT, int U>
 hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
   auto kern = fused_kernel<DT, U>;
-  const size_t smem = shared_bytes(pl.S);
+  const size_t smem = shared_bytes(pl.U);
   static int configured_smem = 0;  // attribute is per kernel; raise it once
   if (configured_smem < int(smem)) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) !=
