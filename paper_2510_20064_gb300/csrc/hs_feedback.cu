@@ -1,16 +1,17 @@
 // hs_feedback.cu -- hs_feedback / hs_feedback_path: argument checks and the
 // choice of kernels, plus the two-pass stochastic kernels.
 //
-// Stochastic rows go to the single-read cluster kernel (hs_fused.cu) when it
-// takes them (bf16/fp16, V % 8 == 0, 16-byte-aligned logits, N <= 32, V up to
-// 153600); greedy rows go to the argmax kernels (hs_greedy.cu).  Everything
-// else takes the two-pass path below, which reads each logit twice:
+// Greedy rows go to the argmax kernels (hs_greedy.cu).  Stochastic bf16/fp16
+// rows with V % 8 == 0, 16-byte-aligned logits and N <= 32 go to the
+// single-read cluster kernel (hs_fused.cu) when V <= 153600, else to the
+// persistent streaming kernel (hs_stream.cu).  Everything else takes the
+// two-pass path below, which reads each logit twice:
 //   row_stats_kernel  one CTA per logit row: max and
 //                     S = sum_v 2^{(z_v - m) log2e / T}   (Thm 1's softmax)
 //   overlap_kernel    one CTA per ((b,k) tile, vocab chunk): p_v built once
 //                     and reused for all N drafters, sum_v min(p_v, q_{i,v})
 //                     (Thm 1), one partial sum per chunk
-//   finalize_kernel   one thread per (i,b): alpha over the P positions from
+//   finalize_kernel   one warp per (i,b): alpha over the P positions from
 //                     the partials in a fixed order, then e_len (Thm 3).
 #include <math.h>
 #include <stdint.h>
@@ -20,6 +21,7 @@
 #include "hs_common.cuh"
 #include "hs_fused.h"
 #include "hs_greedy.h"
+#include "hs_stream.h"
 
 namespace hs {
 
@@ -238,6 +240,11 @@ Layout layout(int N, int B, int P, int V, int dtype, int greedy) {
   L.partial_off = align256(size_t(rows) * sizeof(RowStat));
   const size_t partial = size_t(B) * P * L.nchunk * size_t(N) * sizeof(float);
   L.total = L.partial_off + align256(partial);
+  // the streaming kernel's workspace, when it may take the call
+  if (stream::eligible_sizes(dtype, N, V, greedy)) {
+    const size_t ss = align256(stream::workspace_bytes(N, B, P, V));
+    if (ss > L.total) L.total = ss;
+  }
   return L;
 }
 
@@ -303,6 +310,9 @@ hs_status feedback_common(const void* target, const int32_t* path, int M, const 
   if (fused::eligible(target, drafter, dtype, N, V, greedy))
     return fused::launch(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, dev_status,
                          s);
+  if (stream::eligible(target, drafter, dtype, N, V, greedy))
+    return stream::launch(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, ws,
+                          dev_status, s);
   switch (dtype) {
     case HS_BF16:
       return dispatch_vec<HS_BF16>(vec, target, path, M, drafter, N, B, P, V, c, alpha, e_len,
@@ -329,6 +339,7 @@ extern "C" int hs_feedback_kernel_count(int N, int B, int P, int V, int dtype, i
   if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return 0;
   if (!hs::sizes_ok(N, B, P, V)) return 0;
   if (hs::fused::eligible_sizes(dtype, N, V, greedy)) return 2;  // 16-byte-aligned logits
+  if (hs::stream::eligible_sizes(dtype, N, V, greedy)) return 2;
   return greedy ? 2 : 3;
 }
 

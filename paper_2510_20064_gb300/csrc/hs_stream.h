@@ -1,0 +1,31 @@
+// hs_stream.h -- internal interface of the persistent single-DRAM-read
+// stochastic feedback kernel (hs_stream.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "hedgefb.h"
+
+namespace hs {
+namespace stream {
+
+// Sizes and mode the kernel takes (pointer alignment aside).
+bool eligible_sizes(int dtype, int N, int V, int greedy);
+
+// Same, plus the 16-byte alignment of both logit tensors.
+bool eligible(const void* target, const void* drafter, int dtype, int N, int V, int greedy);
+
+// Workspace: per-chunk row statistics, alpha partials and tile counters.
+size_t workspace_bytes(int N, int B, int P, int V);
+
+// alpha [N,B,P] (and e_len [N,B] when non-null); c = log2(e) / T.  Clears
+// the tile counters, launches the persistent kernel and, for e_len, one
+// small kernel.
+hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
+                 int N, int B, int P, int V, float c, float* alpha, float* e_len, void* ws,
+                 int* dev_status, cudaStream_t stream);
+
+}  // namespace stream
+}  // namespace hs

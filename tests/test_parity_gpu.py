@@ -230,11 +230,12 @@ def test_full_size_greedy_everything():
 
 # ---- both feedback paths ------------------------------------------------------
 # bf16/fp16 rows with V % 8 == 0, 16-byte-aligned logits and N <= 32 take the
-# single-read cluster kernel (cluster size 1, 2, 4 or 8 by V); everything
-# else takes the two-pass kernels.  These cases cross each boundary.
+# single-read cluster kernel (cluster size 1, 2, 4 or 8 by V) up to
+# V = 153600 and the persistent streaming kernel above; everything else takes
+# the two-pass kernels.  These cases cross each boundary.
 
 @pytest.mark.parametrize("V", [8, 4096, 19200, 19208, 38400, 38408, 76800, 76808, 128256,
-                               151936, 153600, 153608])
+                               151936, 153600, 153608, 262144])
 def test_cluster_sizes(V):
     w = synth.Workload("vsweep", N=3, B=2, P=3, V=V, dtype="bf16", temperature=0.8,
                        target="zipf", sigma="qwen")
@@ -268,3 +269,20 @@ def test_fp16_full_vocab():
     d = synth.make_inputs(w, device=DEV, seed=11)
     compare_full(d, 0.7, False)
     compare_full(d, 0.7, True)
+
+
+def test_streaming_kernel_many_tiles():
+    """V above the cluster kernel's range with many tiles per CTA."""
+    w = synth.Workload("big_vocab", N=5, B=24, P=4, V=200000, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=21)
+    a, e, st = run(d, 0.9, False)
+    assert st == 0
+    rng = np.random.default_rng(4)
+    samples = [(int(rng.integers(5)), int(rng.integers(24)), int(rng.integers(4)))
+               for _ in range(30)]
+    ref = oracle_alpha_rows(d, samples, 0.9, False)
+    assert_rel(np.array([a[s] for s in samples]), ref, RTOL_ALPHA, "streaming alpha")
+    col = oracle_alpha_rows(d, [(2, 7, k) for k in range(4)], 0.9, False)
+    assert_rel(np.array([e[2, 7]]), np.array([1.0 + np.cumprod(col[:-1]).sum()]), RTOL_ALPHA,
+               "streaming e_len")
