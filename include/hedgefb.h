@@ -105,6 +105,33 @@ hs_status hs_feedback(const void* target, const void* drafter, int dtype, int N,
                       float* alpha, float* e_len, void* workspace,
                       size_t workspace_bytes, int* dev_status, void* stream);
 
+/* Bytes of the fixed device scratch behind hs_feedback_static. */
+#define HS_STATIC_SCRATCH_BYTES (16u << 20)
+
+/* hs_feedback without a workspace argument, for callers that cannot
+ * allocate device memory at call time: a serving loop whose memory is
+ * reserved up front by another allocator, or code that must not pay for (or
+ * synchronise on) cudaMalloc while requests are in flight.  Same arguments
+ * and results as hs_feedback, minus `workspace` / `workspace_bytes`.  The
+ * paper has no counterpart; this is a deployment convenience.
+ *  - The kernels that need scratch (greedy argmax partials, the streaming
+ *    and two-pass stochastic paths) use a fixed array of
+ *    HS_STATIC_SCRATCH_BYTES bytes compiled into the library; every GPU that
+ *    loads the library keeps it until the process exits.  The call makes no
+ *    cudaMalloc, cudaFree or other allocating call.
+ *  - Sizes whose hs_feedback_workspace_size exceeds HS_STATIC_SCRATCH_BYTES
+ *    return HS_ERR_UNSUPPORTED before any launch.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current); make that first call
+ *    before capturing a stream into a CUDA graph.
+ *  - Every call on a device shares the one array, which keeps the last
+ *    call's contents; whatever must start at zero is cleared by the call
+ *    itself.  Calls whose executions overlap on the GPU (different streams,
+ *    or graphs replayed concurrently) race on it: order them. */
+hs_status hs_feedback_static(const void* target, const void* drafter, int dtype, int N,
+                             int B, int P, int V, float temperature, int greedy,
+                             float* alpha, float* e_len, int* dev_status, void* stream);
+
 /* As hs_feedback, but the target rows come from a draft tree (Sec. 2.3,
  * Fig. "illus_gamma"): row k of query b is tree_target[b, path_idx[b,k], :].
  *   tree_target  device, [B,M,V] logits at the M tree nodes of each query.

@@ -35,6 +35,7 @@ SIGNATURES = {
     "hs_feedback_kernel_count": ([_I, _I, _I, _I, _I, _I], _I),
     "hs_feedback": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
+    "hs_feedback_static": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _P], _I),
     "hs_hedge_update": ([_P, _I, _I, _F, _P, _P, _P], _I),
     "hs_normalhedge_update": ([_P, _P, _P, _I, _I, _P, _P], _I),
     "hs_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P], _I),
@@ -117,7 +118,7 @@ def hs_feedback_kernel_count(N: int, B: int, P: int, V: int, dtype, greedy: bool
     return int(lib().hs_feedback_kernel_count(N, B, P, V, code, int(bool(greedy))))
 
 
-def _feedback_outputs(drafter, alpha, e_len, workspace, greedy):
+def _feedback_outputs(drafter, alpha, e_len, workspace, greedy, with_workspace=True):
     N, B, P, V = drafter.shape
     dev = drafter.device
     if alpha is None:
@@ -126,6 +127,8 @@ def _feedback_outputs(drafter, alpha, e_len, workspace, greedy):
         e_len = torch.empty((N, B), device=dev, dtype=torch.float32)
     _need(alpha, "alpha", torch.float32, (N, B, P))
     _need(e_len, "e_len", torch.float32, (N, B))
+    if not with_workspace:
+        return alpha, e_len, None, 0
     ws_bytes = hs_feedback_workspace_size(N, B, P, V, drafter.dtype, greedy)
     if workspace is None and ws_bytes > 0:
         workspace = torch.empty(ws_bytes, device=dev, dtype=torch.uint8)
@@ -146,6 +149,21 @@ def hs_feedback(target: torch.Tensor, drafter: torch.Tensor, temperature: float 
                            _ptr(workspace), ws_bytes if workspace is not None else 0,
                            _ptr(dev_status), _stream(stream))
     _check(st, "hs_feedback")
+    return alpha, e_len
+
+
+def hs_feedback_static(target: torch.Tensor, drafter: torch.Tensor, temperature: float = 1.0,
+                       greedy: bool = False, alpha=None, e_len=None, dev_status=None, stream=None):
+    """hs_feedback with its scratch in the library's fixed device array
+    (nothing is allocated by the call; see include/hedgefb.h)."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(target, "target", drafter.dtype, (B, P, V))
+    alpha, e_len, _, _ = _feedback_outputs(drafter, alpha, e_len, None, greedy, with_workspace=False)
+    st = lib().hs_feedback_static(_ptr(target), _ptr(drafter), _dtype_code(drafter), N, B, P, V,
+                                  float(temperature), int(bool(greedy)), _ptr(alpha), _ptr(e_len),
+                                  _ptr(dev_status), _stream(stream))
+    _check(st, "hs_feedback_static")
     return alpha, e_len
 
 
