@@ -51,6 +51,9 @@ def parse_args():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--session", action="store_true",
+                    help="long-session learner run: cumulative regret over the workload's rounds")
+    ap.add_argument("--rounds", type=int, default=0, help="session rounds (0: the workload's)")
     return ap.parse_args()
 
 
@@ -173,8 +176,8 @@ def oracle_sample(w, sets, greedy, budget_s=10.0):
     path_np = None if path is None else path.cpu().numpy()
     evals, tiles, t_used = 0, 0, 0.0
     tile = 0
-    while t_used < budget_s and tile < w.B * w.P:
-        b, k = divmod(tile, w.P)
+    while t_used < budget_s:
+        b, k = divmod(tile % (w.B * w.P), w.P)
         trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
         drows = synth.storage_numpy(d["drafter"][:, b, k])
         t0 = time.perf_counter()
@@ -185,8 +188,9 @@ def oracle_sample(w, sets, greedy, budget_s=10.0):
         tiles += 1
         tile += 1
     return {"value": evals / t_used, "unit": "evals/s", "cores": 1, "kind": "oracle",
-            "sample": f"{tiles} of {w.B * w.P} (b,k) tiles x {w.N} drafters x V={w.V} of the "
-                      f"{w.name} workload, fp64 C oracle, 1 thread, {t_used:.1f} s"}
+            "sample": f"{tiles} (b,k) tiles (cycling over the {w.B * w.P} of one input set) x "
+                      f"{w.N} drafters x V={w.V} of the {w.name} workload, fp64 C oracle, "
+                      f"1 thread, {t_used:.1f} s"}
 
 
 # ---- the benchmark -------------------------------------------------------------
@@ -403,8 +407,72 @@ def run_reference(args):
     }), flush=True)
 
 
+def run_session(args):
+    """Many verification rounds with fresh logits each round: feedback, then
+    Hedge and NormalHedge side by side on the same losses; reports the mean
+    over queries of the cumulative regret sum_t f_t[i_t] - min_i sum_t f_t[i]
+    (Sec. 3.1) of each learner."""
+    import torch
+
+    import paper_2510_20064_gb300 as hf
+    from paper_2510_20064_gb300 import synth
+    w = synth.WORKLOADS["long_session" if args.workload == DEFAULT_WORKLOAD else args.workload]
+    rounds = args.rounds or w.rounds
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    hf.lib()
+    N, B, P = w.N, w.B, w.P
+    eta = w.eta or math.sqrt(8 * math.log(max(N, 2)) / rounds)
+    alpha = torch.empty(N, B, P, device=dev)
+    e_len = torch.empty(N, B, device=dev)
+    ws = torch.empty(max(1, hf.hs_feedback_workspace_size(N, B, P, w.V, synth.DTYPES[w.dtype],
+                                                          False)), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    learners = {}
+    for name, kind in (("hedge", hf.HS_HEDGE), ("normalhedge", hf.HS_NORMALHEDGE)):
+        learners[name] = dict(kind=kind, state=torch.zeros(N, B, device=dev),
+                              weights=torch.full((N, B), 1.0 / N, device=dev),
+                              sel=torch.zeros(B, dtype=torch.int32, device=dev),
+                              played=torch.zeros(B, device=dev),
+                              loss=torch.empty(N, B, device=dev))
+    cum = torch.zeros(N, B, device=dev, dtype=torch.float64)
+    t_fb = 0.0
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start = time.time()
+    for t in range(rounds):
+        d = synth.make_inputs(w, rnd=t, device=dev)
+        ev0.record()
+        hf.hs_feedback(d["target"], d["drafter"], w.temperature, False, alpha=alpha, e_len=e_len,
+                       workspace=ws, dev_status=status)
+        for L in learners.values():
+            hf.hs_learner_step(alpha, e_len, hf.HS_LOSS_LENGTH, L["kind"], eta, L["state"],
+                               L["weights"], L["sel"], loss_out=L["loss"],
+                               played_loss=L["played"])
+        ev1.record()
+        cum += learners["hedge"]["loss"].double()
+        ev1.synchronize()
+        t_fb += ev0.elapsed_time(ev1)
+        del d
+    assert int(status.item()) == 0, hf.hs_status_string(int(status.item()))
+    best = cum.min(dim=0).values
+    out = {"session": w.name, "rounds": rounds, "N": N, "B": B, "K": w.K, "V": w.V,
+           "eta_hedge": eta, "ms_per_round_feedback_and_learners": t_fb / rounds,
+           "wall_s": time.time() - t_start}
+    for name, L in learners.items():
+        reg = (L["played"].double() - best)
+        out[f"{name}_regret_mean"] = float(reg.mean())
+        out[f"{name}_regret_max"] = float(reg.max())
+        out[f"{name}_final_choice_is_expert_frac"] = float(
+            (L["sel"].long().cpu() == (torch.arange(B) + (rounds - 1) // 250) % N).float().mean())
+    out["best_fixed_drafter_loss_mean"] = float(best.mean())
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse_args()
+    if args.session:
+        run_session(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:
