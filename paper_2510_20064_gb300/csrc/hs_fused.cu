@@ -7,27 +7,26 @@
 // cluster of C CTAs takes one (b,k) tile, each CTA a V/C slice, and loops
 // persistently over tiles:
 //   * the CTA's slice of every row of its tiles -- the target row, then the
-//     N drafter rows -- streams into a 3-stage shared-memory ring with
-//     cp.async.bulk (TMA; each CTA reads its own slice, no multicast); a
-//     coordinator warp refills a stage as soon as every consumer has read it;
+//     N drafter rows -- streams into a kStages-deep shared-memory ring with
+//     cp.async.bulk (TMA; each CTA reads its own slice, no multicast);
 //   * 15 consumer warps load a row from the ring into registers, form
 //     e_v = 2^{z_v c - o_w} with o_w = c * (the warp's max), c = log2e/T,
-//     and their sum (one ex2 per logit, values kept in registers);
-//   * the cluster merges the per-CTA (offset, sum) pairs through distributed
-//     shared memory: every CTA stores its pair into each peer and arrives on
-//     the peer's mbarrier; then every thread knows the row's offset O and
-//     normaliser Z, and p_v or q_v = e_v 2^{o_t - O} / Z;
-//   * the target's p stays in shared memory (fp32) for the tile's N drafters;
-//     a drafter row adds sum_v min(p_v, q_v) to its per-warp partial;
-//   * at the end of a tile the coordinator sums the warps' N partials and
-//     sends them to the cluster's rank 0, whose coordinator sums them in rank
-//     order and writes alpha[:, b, k] one tile later.  The coordinator never
-//     blocks: its waits poll, servicing ring refills meanwhile, and no
-//     consumer warp waits for another warp of its CTA.
-// Rows are software-pipelined: the pass over row g+1's logits runs while
-// row g's cluster exchange is in flight, so each thread holds two rows of
-// exponentials (eA / eB).  Every wait is bounded; on expiry the kernel
-// records HS_ERR_TIMEOUT and finishes without waiting further.
+//     and their sum (one ex2 per logit), and park the exponentials in
+//     tensor memory (TMEM), each thread in its own lane;
+//   * a coordinator warp merges the 15 warps' (offset, sum) pairs of a row,
+//     stores the CTA's pair into every peer CTA (distributed shared memory)
+//     and arrives on the peer's mbarrier, and refills the row's ring stage;
+//     every consumer thread then merges the C pairs into the row's offset O
+//     and normaliser Z, so p_v or q_v = e_v 2^{o_w - O} / Z;
+//   * the target's p goes to TMEM for the tile's N drafters; a drafter row
+//     adds sum_v min(p_v, q_v) to its per-warp partial;
+//   * the coordinator sums each tile's per-warp partials and sends them to
+//     the cluster's rank 0, whose coordinator sums them in rank order and
+//     writes alpha[:, b, k] one tile later.
+// Rows are software-pipelined three deep: pass 1 of row g+2 runs before
+// pass 2 of row g, so a row's exchange has two rows of work to hide behind.
+// Every wait is bounded; on expiry the kernel records HS_ERR_TIMEOUT and
+// finishes without waiting further.
 #include <math.h>
 #include <stdint.h>
 
@@ -38,19 +37,16 @@ namespace hs {
 namespace fused {
 namespace {
 
-// 15 consumer warps + 1 load warp: 16 warps put 4 on each SM sub-partition,
-// which leaves 128 registers per thread for the two rows of exponentials a
-// consumer thread keeps.
+// 15 consumer warps + 1 coordinator warp: 16 warps put 4 on each SM
+// sub-partition and 128 registers per thread; each consumer thread keeps
+// p and two rows of exponentials (3 x 8U columns) in TMEM.
 constexpr int kConsumerWarps = 15;
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;
-constexpr int kStages = 3;
-// Rows ahead of the ring whose slice is prefetched into L2 (bulk prefetch,
-// no shared memory): the ring's TMA loads then hit L2, which keeps a few
-// hundred KB per SM in flight although only ~2 stages fit next to p.
-constexpr int kPrefetch = 0;
-constexpr int kXSlots = 4;  // rows whose exchange may be in flight at once
-constexpr int kASlots = 4;  // tiles whose alpha partials may be in flight
+constexpr int kStages = 4;
+constexpr int kXSlots = 8;  // rows whose exchange may be in flight at once
+constexpr int kASlots = 8;  // tiles whose alpha partials may be in flight (rank 0)
+constexpr int kTSlots = 4;  // tiles whose per-warp partials await the coordinator
 constexpr int kMaxU = 5;    // 16-byte vectors per consumer thread and row
 constexpr long long kTimeoutCycles = 1LL << 31;  // about a second
 constexpr uint32_t kNegInfBf16x2 = 0xFF80FF80u;
@@ -58,18 +54,18 @@ constexpr uint32_t kNegInfF16x2 = 0xFC00FC00u;
 
 struct __align__(16) Shared {
   uint64_t full[kStages];          // ring stage loaded (TMA complete_tx)
-  uint64_t empty[kStages];         // ring stage read by every consumer warp
   uint64_t redbar[kXSlots];        // every consumer warp posted its row pair
   uint64_t xbar[kXSlots];          // every rank's pair of a row arrived
-  uint64_t accbar[2];              // every consumer warp posted a tile's partials
+  uint64_t accbar[kTSlots];        // every consumer warp posted a tile's partials
   uint64_t abar[kASlots];          // every rank's tile partials arrived (rank 0)
   float2 red[kXSlots][16];                // per-warp (offset, sum) of a row
   float2 xch[kXSlots][kMaxC];             // per-rank (offset, sum) of a row
-  float acc[2][kMaxN][kConsumerWarps];    // per-warp alpha partials of a tile
-  uint32_t tvalid[2];                     // the tile's target row is usable
-  uint32_t dvalid[2];                     // bit i: drafter i's row is usable
+  float acc[kTSlots][kMaxN][kConsumerWarps];  // per-warp alpha partials of a tile
+  uint32_t tvalid[kTSlots];               // the tile's target row is usable
+  uint32_t dvalid[kTSlots];               // bit i: drafter i's row is usable
   float clacc[kASlots][kMaxC][kMaxN];     // per-rank alpha partials (rank 0)
   int error;
+  uint32_t tmem_base;  // tensor memory: p and two rows of exponentials per thread
 };
 
 struct Params {
@@ -139,14 +135,6 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
                "[%0], [%1], %2, [%3];"
                :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_probe(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile("{\n\t.reg .pred p;\n\t"
-               "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-               "selp.u32 %0, 1, 0, p;\n\t}"
-               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
-  return ok != 0;
 }
 // Arrive on a barrier in another CTA of the cluster, ordering this thread's
 // earlier shared::cluster stores before the arrival.
@@ -240,6 +228,64 @@ __device__ __forceinline__ f2_t fmul2(f2_t a, f2_t b) {
   return r;
 }
 
+// ---- tensor memory ------------------------------------------------------------
+// Each consumer thread keeps, in its own TMEM lane, the target's p for its
+// positions and the exponentials of two rows (one 32-bit column per value):
+// the register file then only holds the row being computed.
+__device__ __forceinline__ void tmem_alloc512(uint32_t dst_smem) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;"
+               :: "r"(dst_smem) : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc512(uint32_t taddr) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" :: "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tmem_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+// 8 or 16 consecutive columns of this thread's lane, as packed pairs.
+template <int NV>
+__device__ __forceinline__ void tmem_st(uint32_t taddr, const f2_t* v) {
+  float f[2 * NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) upk(v[i], f[2 * i], f[2 * i + 1]);
+  if (NV == 4)
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};"
+                 :: "r"(taddr), "f"(f[0]), "f"(f[1]), "f"(f[2]), "f"(f[3]), "f"(f[4]),
+                    "f"(f[5]), "f"(f[6]), "f"(f[7]) : "memory");
+  else
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, "
+                 "%9, %10, %11, %12, %13, %14, %15, %16};"
+                 :: "r"(taddr), "f"(f[0]), "f"(f[1]), "f"(f[2]), "f"(f[3]), "f"(f[4]),
+                    "f"(f[5]), "f"(f[6]), "f"(f[7]), "f"(f[8]), "f"(f[9]), "f"(f[10]),
+                    "f"(f[11]), "f"(f[12]), "f"(f[13]), "f"(f[14]), "f"(f[15]) : "memory");
+}
+template <int NV>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, f2_t* v) {
+  float f[2 * NV];
+  if (NV == 4)
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=f"(f[0]), "=f"(f[1]), "=f"(f[2]), "=f"(f[3]), "=f"(f[4]), "=f"(f[5]),
+                   "=f"(f[6]), "=f"(f[7]) : "r"(taddr) : "memory");
+  else
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, "
+                 "%9, %10, %11, %12, %13, %14, %15}, [%16];"
+                 : "=f"(f[0]), "=f"(f[1]), "=f"(f[2]), "=f"(f[3]), "=f"(f[4]), "=f"(f[5]),
+                   "=f"(f[6]), "=f"(f[7]), "=f"(f[8]), "=f"(f[9]), "=f"(f[10]), "=f"(f[11]),
+                   "=f"(f[12]), "=f"(f[13]), "=f"(f[14]), "=f"(f[15]) : "r"(taddr) : "memory");
+#pragma unroll
+  for (int i = 0; i < NV; ++i) v[i] = pk(f[2 * i], f[2 * i + 1]);
+}
+
 // Order-preserving int key of a float (NaN above +inf), so that a warp's
 // maximum is one redux.sync.
 __device__ __forceinline__ int fkey(float f) {
@@ -253,6 +299,22 @@ __device__ __forceinline__ float warp_max_key(float f) {
   return kfloat(__reduce_max_sync(0xffffffffu, fkey(f)));
 }
 
+// Warp maximum, NaN if any lane holds a NaN (sm_100+ redux on f32).
+__device__ __forceinline__ float warp_max_f(float f) {
+  float r;
+  asm volatile("redux.sync.max.NaN.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(f));
+  return r;
+}
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
 // Merge (offset o, sum s) pairs held by the lanes of a warp: the largest
 // offset O (NaN wins, -inf means "no finite logit") and sum_l s_l 2^{o_l - O}.
 __device__ __forceinline__ void warp_merge(float& o, float& s) {
@@ -265,51 +327,55 @@ __device__ __forceinline__ void warp_merge(float& o, float& s) {
 
 // ---- the kernel ---------------------------------------------------------------
 
-template <int DT, int U>
-struct Row {
-  f2_t e[U * 4];  // exponentials of the thread's logits, packed in pairs
-  float o_used;   // offset the exponentials are relative to (the warp's)
-  float o;        // reported offset: -inf when the warp saw no finite logit
+// The coordinator's walk over the global addresses of this CTA's slices of
+// its rows, in stream order: per tile, the target row, then the N drafter
+// rows.  One division per tile; the tree path index of the next tile is
+// fetched a tile ahead.
+struct RowWalk {
+  int r = 0;             // row within the tile
+  int64_t tile = 0;      // global tile index b * P + k
+  const char* tsrc;      // target row slice of the current tile
+  const char* dsrc;      // drafter 0's row slice of the current tile
+  int64_t dstride;       // bytes from drafter i's row to drafter i+1's
+  int next_path = 0;     // path index of the next tile (tree targets)
+
+  __device__ void start_tile(const Params& p, int64_t slice0, int nd) {
+    const int64_t b = tile / p.P, k = tile - b * p.P;
+    const int64_t trow = p.path ? b * p.M + ((nd < 0 || nd >= p.M) ? 0 : nd) : tile;
+    tsrc = static_cast<const char*>(p.target) + (trow * p.V + slice0) * 2;
+    dsrc = static_cast<const char*>(p.drafter) + ((b * p.P + k) * p.V + slice0) * 2;
+  }
+  __device__ void init(const Params& p, uint32_t cid, uint32_t ncl, int64_t slice0) {
+    tile = cid;
+    dstride = int64_t(p.B) * p.P * p.V * 2;
+    const int nd = (p.path && tile < p.ntiles) ? p.path[tile] : 0;
+    if (p.path && tile + ncl < p.ntiles) next_path = p.path[tile + ncl];
+    if (tile < p.ntiles) start_tile(p, slice0, nd);
+  }
+  // source of the current row; then advance
+  __device__ const char* next(const Params& p, uint32_t ncl, int64_t slice0) {
+    const char* src = r == 0 ? tsrc : dsrc + (r - 1) * dstride;
+    if (++r == p.N + 1) {
+      r = 0;
+      tile += ncl;
+      if (tile < p.ntiles) {
+        const int nd = next_path;
+        if (p.path && tile + ncl < p.ntiles) next_path = p.path[tile + ncl];
+        start_tile(p, slice0, nd);
+      }
+    }
+    return src;
+  }
 };
 
-// Global address of this CTA's slice of its row g: row g % (N+1) of the
-// CTA's (g / (N+1))-th tile -- the target row, then the drafter rows.
-__device__ __forceinline__ const char* row_slice(const Params& p, int g, uint32_t cid,
-                                                 uint32_t ncl, int64_t slice0) {
-  const int R = p.N + 1;
-  const int j = g / R, r = g % R;
-  const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
-  const int64_t b = tile / p.P, k = tile % p.P;
-  int64_t row;
-  const void* base;
-  if (r == 0) {
-    if (p.path) {
-      const int nd = p.path[tile];
-      row = b * p.M + ((nd < 0 || nd >= p.M) ? 0 : nd);
-    } else {
-      row = tile;
-    }
-    base = p.target;
-  } else {
-    row = (int64_t(r - 1) * p.B + b) * p.P + k;
-    base = p.drafter;
-  }
-  return static_cast<const char*>(base) + (row * p.V + slice0) * 2;
-}
-
-// Stream row g into `stage` (one thread); with kPrefetch > 0 also prefetch
-// row g + kPrefetch into L2.
-__device__ __forceinline__ void issue(const Params& p, Shared& sh, unsigned char* stage, int g,
-                                      int G, uint32_t cid, uint32_t ncl, int64_t slice0,
+// Stream one row slice into `stage` (one thread).
+__device__ __forceinline__ void issue(Shared& sh, unsigned char* stage, int g, const char* src,
                                       uint32_t bytes) {
   const uint32_t full = saddr(&sh.full[g % kStages]);
   if (bytes) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     mbar_arrive_tx(full, bytes);
-    bulk_load(saddr(stage), row_slice(p, g, cid, ncl, slice0), bytes, full);
-    if (kPrefetch > 0 && g + kPrefetch < G)
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
-                   :: "l"(row_slice(p, g + kPrefetch, cid, ncl, slice0)), "r"(bytes) : "memory");
+    bulk_load(saddr(stage), src, bytes, full);
   } else {
     mbar_arrive(full);
   }
@@ -319,16 +385,12 @@ template <int DT, int U>
 __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Shared& sh = *reinterpret_cast<Shared*>(smem_raw);
-  // every buffer holds SU = U * kConsumers * 8 >= S elements so that each
-  // consumer thread always handles U whole 16-byte vectors; the part past
-  // the CTA's slice is -inf in the ring and 0 in p (set once, below)
+  // every ring stage holds SU = U * kConsumers * 8 >= S elements so that
+  // each consumer thread always handles U whole 16-byte vectors; the part
+  // past the CTA's slice is -inf (set once, below)
   constexpr int SU = U * kConsumers * 8;
   constexpr uint32_t stage_bytes = SU * 2;
   unsigned char* ring = smem_raw + ((sizeof(Shared) + 127) & ~size_t(127));
-  // p of the tile's target, as two planes of float4 so that consecutive
-  // threads read consecutive 16 bytes: pA[vi] = p[8vi..8vi+3], pB[vi] = p[8vi+4..8vi+7]
-  float4* pA = reinterpret_cast<float4*>(ring + kStages * stage_bytes);
-  float4* pB = pA + SU / 8;
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -350,66 +412,48 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     for (int e = len / 2 + tid; e < SU / 2; e += kThreads)
       for (int s = 0; s < kStages; ++s)
         reinterpret_cast<uint32_t*>(ring + s * stage_bytes)[e] = neg;
-    for (int vi = len / 8 + tid; vi < SU / 8; vi += kThreads)
-      pA[vi] = pB[vi] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(saddr(&sh.full[s]), 1);
-      mbar_init(saddr(&sh.empty[s]), kConsumerWarps);
-    }
+    for (int s = 0; s < kStages; ++s) mbar_init(saddr(&sh.full[s]), 1);
     for (int x = 0; x < kXSlots; ++x) {
       mbar_init(saddr(&sh.redbar[x]), kConsumerWarps);
       mbar_init(saddr(&sh.xbar[x]), C);
     }
-    for (int a = 0; a < 2; ++a) mbar_init(saddr(&sh.accbar[a]), kConsumerWarps);
+    for (int a = 0; a < kTSlots; ++a) mbar_init(saddr(&sh.accbar[a]), kConsumerWarps);
     for (int a = 0; a < kASlots; ++a) mbar_init(saddr(&sh.abar[a]), C * N);
     sh.error = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (warp == 0) tmem_alloc512(saddr(&sh.tmem_base));
+  tmem_fence_before();
   cluster_sync_all();
+  tmem_fence_after();
 
   if (warp == kConsumerWarps) {
     // ---------------------------- coordinator -----------------------------
-    // Never blocks: every wait polls its barrier and, while it does, lane 0
-    // refills each ring stage as soon as all consumer warps have read it.
-    // The warp merges the consumer warps' row pairs and sends the CTA's pair
-    // to every rank, and reduces each tile's alpha partials (rank 0 also
-    // writes alpha, one tile late).
-    int issued = 0;
-    auto service = [&]() {
-      if (lane != 0) return;
-      while (issued < G &&
-             (issued < kStages ||
-              mbar_probe(saddr(&sh.empty[issued % kStages]),
-                         uint32_t((issued / kStages) - 1) & 1u))) {
-        issue(p, sh, ring + (issued % kStages) * stage_bytes, issued, G, cid, ncl, slice0, bytes);
-        ++issued;
-      }
-    };
-    auto poll = [&](uint32_t bar, uint32_t parity) {
-      service();
-      const long long t0 = clock64();
-      while (!mbar_probe(bar, parity)) {
-        service();
-        if (*reinterpret_cast<volatile int*>(&sh.error)) return;
-        if (clock64() - t0 > kTimeoutCycles) {
-          *reinterpret_cast<volatile int*>(&sh.error) = 1;
-          report(p.dev_status, HS_ERR_TIMEOUT);
-          return;
-        }
-        __nanosleep(32);
-      }
-    };
+    // Per row g: waits until every consumer warp posted its pass-1 pair (so
+    // the row's ring stage has been read), refills that stage with row
+    // g + kStages, merges the warps' pairs and sends the CTA's pair to every
+    // rank.  Tile j's per-warp alpha partials are complete once row
+    // (j+1)(N+1) + 2 is posted (the consumers run pass 1 two rows ahead of
+    // pass 2); they are then summed and sent to rank 0, which writes alpha
+    // one tile late.  Every wait sleeps in mbarrier try_wait (bounded).
+    RowWalk walk;
+    if (lane == 0) {
+      walk.init(p, cid, ncl, slice0);
+      for (int g = 0; g < G && g < kStages; ++g)
+        issue(sh, ring + g * stage_bytes, g, walk.next(p, ncl, slice0), bytes);
+    }
     auto finish = [&](int j) {  // rank 0: alpha[:, b, k] of tile j
-      poll(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u);
+      wait_phase(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u, sh, p.dev_status);
       if (lane < N) {
         const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
         const int64_t b = tile / P, k = tile % P;
         float t = 0.f;
         for (uint32_t rr = 0; rr < C; ++rr) t += sh.clacc[j % kASlots][rr][lane];
         const bool bad_path = p.path && (p.path[tile] < 0 || p.path[tile] >= p.M);
-        if (bad_path || !sh.tvalid[j & 1] || !((sh.dvalid[j & 1] >> lane) & 1u)) {
+        const int ts = j % kTSlots;
+        if (bad_path || !sh.tvalid[ts] || !((sh.dvalid[ts] >> lane) & 1u)) {
           t = __int_as_float(0x7fc00000);
           report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
         }
@@ -417,18 +461,23 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       }
     };
     auto reduce_tile = [&](int j) {  // tile j's partials -> rank 0
-      poll(saddr(&sh.accbar[j & 1]), uint32_t(j >> 1) & 1u);
+      const int ts = j % kTSlots;
+      wait_phase(saddr(&sh.accbar[ts]), uint32_t(j / kTSlots) & 1u, sh, p.dev_status);
       if (lane < N) {
         float t = 0.f;
-        for (int w = 0; w < kConsumerWarps; ++w) t += sh.acc[j & 1][lane][w];
+        for (int w = 0; w < kConsumerWarps; ++w) t += sh.acc[ts][lane][w];
         st_cluster_f(mapa(saddr(&sh.clacc[j % kASlots][rank][lane]), 0), t);
         mbar_arrive_remote(mapa(saddr(&sh.abar[j % kASlots]), 0));
       }
       if (rank == 0 && j > 0) finish(j - 1);  // long since complete
     };
+    int reduced = 0;  // tiles sent to rank 0
     for (int g = 0; g < G; ++g) {
       const int x = g % kXSlots;
-      poll(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u);
+      wait_phase(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
+      if (lane == 0 && g + kStages < G)
+        issue(sh, ring + (g % kStages) * stage_bytes, g + kStages, walk.next(p, ncl, slice0),
+              bytes);
       float2 v = lane < kConsumerWarps ? sh.red[x][lane] : make_float2(-INFINITY, 0.f);
       float oc = v.x, sc = v.y;
       warp_merge(oc, sc);
@@ -436,16 +485,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
         st_cluster_f2(mapa(saddr(&sh.xch[x][rank]), lane), oc, sc);
         mbar_arrive_remote(mapa(saddr(&sh.xbar[x]), lane));
       }
-      // tile j's partials are posted after the consumers' pass over the
-      // first row of tile j+1, so reduce tile j once that row is merged
-      if (g % R == 0 && g > 0) reduce_tile(g / R - 1);
+      while (reduced < my_tiles && (reduced + 1) * R + 2 <= g) reduce_tile(reduced++);
     }
-    if (G > 0) {
-      reduce_tile(my_tiles - 1);
-      if (rank == 0) finish(my_tiles - 1);
-    }
-    // every row was issued (the consumers have read them all); drain: every
-    // copy has landed before the CTA may exit
+    while (reduced < my_tiles) reduce_tile(reduced++);
+    if (G > 0 && rank == 0) finish(my_tiles - 1);
+    // drain: every copy has landed before the CTA may exit
     if (lane == 0)
       for (int g = max(0, G - kStages); g < G; ++g)
         wait_phase(saddr(&sh.full[g % kStages]), uint32_t(g / kStages) & 1u, sh, p.dev_status,
@@ -454,23 +498,29 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     // ------------------------------ consumers -----------------------------
     const float c = p.c;
     uint32_t tvalid = 0, dvalid = 0;  // target row usable; bit i: drafter i usable
-    Row<DT, U> A, Bv;
+    // the last vector round holds the slice's tail: warps whose vectors there
+    // all lie past the slice skip it (they would only see the -inf padding)
+    const bool tail = (U - 1) * kConsumers + warp * 32 < len / 8;
+    // this thread's TMEM lane (the warp's quadrant) and columns: [0, 8U) p of
+    // the tile's target, [8U (1+s), 8U (2+s)) the exponentials of row slot s
+    const uint32_t tbase = sh.tmem_base + (uint32_t(32 * (warp & 3)) << 16) +
+                           uint32_t((warp >> 2) * 3 * U * 8);
 
     // pass 1: load row g from the ring (then release the stage); warp max;
-    // exponentials relative to the warp's offset, kept in registers; post
-    // the warp's (offset, sum) for the coordinator
-    auto pass1 = [&](int g, Row<DT, U>& Rw) {
+    // exponentials relative to the warp's offset; post the warp's (offset,
+    // sum) for the coordinator.  E keeps the exponentials (packed pairs).
+    auto pass1 = [&](int g, f2_t (&E)[U * 4], float& o, float& o_used) {
       const int s = g % kStages;
       wait_phase(saddr(&sh.full[s]), uint32_t(g / kStages) & 1u, sh, p.dev_status);
       const uint32_t stage = saddr(ring + s * stage_bytes);
       uint32_t w[U * 4];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const uint4 v = lds128(stage + (u * kConsumers + tid) * 16);
+        uint4 v = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+        if (DT != HS_BF16) v = make_uint4(kNegInfF16x2, kNegInfF16x2, kNegInfF16x2, kNegInfF16x2);
+        if (u < U - 1 || tail) v = lds128(stage + (u * kConsumers + tid) * 16);
         w[4 * u] = v.x; w[4 * u + 1] = v.y; w[4 * u + 2] = v.z; w[4 * u + 3] = v.w;
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(saddr(&sh.empty[s]));
       uint32_t mx[U * 2];  // pairwise tree: log-depth dependency chain
 #pragma unroll
       for (int q = 0; q < U * 2; ++q) mx[q] = pmax<DT>(w[2 * q], w[2 * q + 1]);
@@ -478,58 +528,92 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       for (int d = 1; d < U * 2; d *= 2)
 #pragma unroll
         for (int q = 0; q + d < U * 2; q += 2 * d) mx[q] = pmax<DT>(mx[q], mx[q + d]);
-      const float m = warp_max_key(max_nan(lo<DT>(mx[0]), hi<DT>(mx[0])));
-      Rw.o = (m == -INFINITY) ? -INFINITY : m * c;
-      Rw.o_used = (m == -INFINITY) ? 0.f : Rw.o;
-      const f2_t cc = pk(c, c), off = pk(-Rw.o_used, -Rw.o_used);
+      const float m = warp_max_f(fmax_nan(lo<DT>(mx[0]), hi<DT>(mx[0])));
+      o = (m == -INFINITY) ? -INFINITY : m * c;
+      o_used = (m == -INFINITY) ? 0.f : o;
+      const f2_t cc = pk(c, c), off = pk(-o_used, -o_used);
       f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
       for (int q = 0; q < U * 4; ++q) {
-        float a, b;
-        upk(ffma2(pk(lo<DT>(w[q]), hi<DT>(w[q])), cc, off), a, b);
-        Rw.e[q] = pk(ex2(a), ex2(b));
-        acc[q & 1] = fadd2(acc[q & 1], Rw.e[q]);
+        if (q < (U - 1) * 4 || tail) {
+          float a, b;
+          upk(ffma2(pk(lo<DT>(w[q]), hi<DT>(w[q])), cc, off), a, b);
+          E[q] = pk(ex2(a), ex2(b));
+          acc[q & 1] = fadd2(acc[q & 1], E[q]);
+        }
       }
       float s0, s1, s2, s3;
       upk(acc[0], s0, s1);
       upk(acc[1], s2, s3);
       const float sum = warp_sum((s0 + s1) + (s2 + s3));
       if (lane == 0) {
-        sh.red[g % kXSlots][warp] = make_float2(Rw.o, sum);
+        sh.red[g % kXSlots][warp] = make_float2(o, sum);
         mbar_arrive(saddr(&sh.redbar[g % kXSlots]));
       }
     };
 
-    // all ranks' pairs of row g: the row's offset O and 1/Z
+    // the exponentials of a row into its TMEM slot, two vectors per store
+    auto store_row = [&](int slot, const f2_t (&E)[U * 4]) {
+      const uint32_t t = tbase + uint32_t((1 + slot) * U * 8);
+#pragma unroll
+      for (int u = 0; u < U; u += 2) {
+        if (u + 1 < U) {
+          if (u + 1 < U - 1 || tail) tmem_st<8>(t + u * 8, &E[4 * u]);
+          else tmem_st<4>(t + u * 8, &E[4 * u]);
+        } else if (tail) {
+          tmem_st<4>(t + u * 8, &E[4 * u]);
+        }
+      }
+    };
+
+    // all ranks' pairs of row g: the row's offset O and 1/Z.  Lane l holds
+    // rank (l & 7)'s pair (neutral past C); a butterfly over each group of 8
+    // lanes leaves the same merged pair in every lane.
     auto gather = [&](int g, float& O, float& invZ) -> bool {
       const int x = g % kXSlots;
       wait_phase(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
-      float2 v = lane < int(C) ? sh.xch[x][lane] : make_float2(-INFINITY, 0.f);
-      float o = v.x, s = v.y;
-      warp_merge(o, s);
+      const int r8 = lane & 7;
+      const float2 v = r8 < int(C) ? sh.xch[x][r8] : make_float2(-INFINITY, 0.f);
+      float o = v.x;
+#pragma unroll
+      for (int d = 1; d < 8; d *= 2) o = fmax_nan(o, __shfl_xor_sync(0xffffffffu, o, d));
+      float t = (v.x == -INFINITY || o == -INFINITY) ? 0.f : v.y * ex2(v.x - o);
+#pragma unroll
+      for (int d = 1; d < 8; d *= 2) t += __shfl_xor_sync(0xffffffffu, t, d);
       O = o;
-      invZ = 1.f / s;
-      return isfinite(o) && s > 0.f;
+      invZ = rcp_approx(t);
+      return isfinite(o) && t > 0.f;
     };
 
-    // pass 2: target -> p into shared memory; drafter i -> alpha partial
-    auto pass2 = [&](int g, Row<DT, U>& Rw) {
-      const int j = g / R, r = g % R;
+    // pass 2 of row g (exponentials in TMEM slot g & 1): target -> p into
+    // TMEM; drafter i -> alpha partial
+    auto pass2 = [&](int g, float o, float o_used) {
+      const int j = g / R, r = g - (g / R) * R;
       float O, invZ;
       const bool ok = gather(g, O, invZ);
-      const float f = (Rw.o == -INFINITY || !ok) ? 0.f : ex2(Rw.o_used - O) * invZ;
+      const float f = (o == -INFINITY || !ok) ? 0.f : ex2(o_used - O) * invZ;
       const f2_t ff = pk(f, f);
+      const uint32_t te = tbase + uint32_t((1 + (g & 1)) * U * 8);
+      tmem_wait_st();  // this row's exponentials and the tile's p have landed
       if (r == 0) {
         tvalid = ok ? 1u : 0u;
         dvalid = 0;
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const int vi = u * kConsumers + tid;
-          float q[8];
+        for (int u = 0; u < U; u += 2) {
+          f2_t e[8];
+          if (u + 1 < U && (u + 1 < U - 1 || tail)) {
+            tmem_ld<8>(te + u * 8, e);
+            tmem_wait_ld();
 #pragma unroll
-          for (int h = 0; h < 4; ++h) upk(fmul2(Rw.e[4 * u + h], ff), q[2 * h], q[2 * h + 1]);
-          pA[vi] = make_float4(q[0], q[1], q[2], q[3]);
-          pB[vi] = make_float4(q[4], q[5], q[6], q[7]);
+            for (int h = 0; h < 8; ++h) e[h] = fmul2(e[h], ff);
+            tmem_st<8>(tbase + u * 8, e);
+          } else if (u + 1 < U || tail) {
+            tmem_ld<4>(te + u * 8, e);
+            tmem_wait_ld();
+#pragma unroll
+            for (int h = 0; h < 4; ++h) e[h] = fmul2(e[h], ff);
+            tmem_st<4>(tbase + u * 8, e);
+          }
         }
         return;
       }
@@ -537,15 +621,29 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       if (ok) dvalid |= 1u << i;
       f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int vi = u * kConsumers + tid;
-        const float4 p0 = pA[vi], p1 = pB[vi];
-        const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+      for (int u = 0; u < U; u += 2) {
+        f2_t e[8], pv[8];
+        int nv = 0;
+        if (u + 1 < U && (u + 1 < U - 1 || tail)) {
+          tmem_ld<8>(te + u * 8, e);
+          tmem_ld<8>(tbase + u * 8, pv);
+          nv = 8;
+        } else if (u + 1 < U || tail) {
+          tmem_ld<4>(te + u * 8, e);
+          tmem_ld<4>(tbase + u * 8, pv);
+          nv = 4;
+        }
+        if (nv) {
+          tmem_wait_ld();
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          float xx, yy;
-          upk(fmul2(Rw.e[4 * u + h], ff), xx, yy);
-          acc[h & 1] = fadd2(acc[h & 1], pk(fminf(pv[2 * h], xx), fminf(pv[2 * h + 1], yy)));
+          for (int h = 0; h < 8; ++h) {
+            if (h < nv) {
+              float xx, yy, pa, pb;
+              upk(fmul2(e[h], ff), xx, yy);
+              upk(pv[h], pa, pb);
+              acc[h & 1] = fadd2(acc[h & 1], pk(fminf(pa, xx), fminf(pb, yy)));
+            }
+          }
         }
       }
       float a0, a1, a2, a3;
@@ -553,37 +651,59 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       upk(acc[1], a2, a3);
       const float a = warp_sum((a0 + a1) + (a2 + a3));
       if (lane == 0) {
-        sh.acc[j & 1][i][warp] = a;
+        const int ts = j % kTSlots;
+        sh.acc[ts][i][warp] = a;
         if (i == N - 1) {  // tile end: hand the partials to the coordinator
           if (warp == 0) {
-            sh.tvalid[j & 1] = tvalid;
-            sh.dvalid[j & 1] = dvalid;
+            sh.tvalid[ts] = tvalid;
+            sh.dvalid[ts] = dvalid;
           }
-          mbar_arrive(saddr(&sh.accbar[j & 1]));
+          mbar_arrive(saddr(&sh.accbar[ts]));
         }
       }
     };
 
-    pass1(0, A);
-    for (int g = 0; g < G; g += 2) {
-      if (g + 1 < G) pass1(g + 1, Bv);
-      pass2(g, A);
-      if (g + 1 < G) {
-        if (g + 2 < G) pass1(g + 2, A);
-        pass2(g + 1, Bv);
+    // three rows in flight: pass 1 of row g+2 runs before pass 2 of row g,
+    // so the cluster exchange of a row has two rows of work to hide behind
+    f2_t E[U * 4];
+    float o0 = 0.f, ou0 = 0.f, o1 = 0.f, ou1 = 0.f;  // offsets of rows in slots 0, 1
+    for (int g = -2; g < G; ++g) {
+      const bool more = g + 2 < G;
+      float on = 0.f, oun = 0.f;
+      if (more) pass1(g + 2, E, on, oun);
+      if (g >= 0) pass2(g, (g & 1) ? o1 : o0, (g & 1) ? ou1 : ou0);
+      if (more) {
+        store_row(g & 1, E);
+        if (g & 1) {
+          o1 = on;
+          ou1 = oun;
+        } else {
+          o0 = on;
+          ou0 = oun;
+        }
       }
     }
   }
-  // no CTA may leave while a peer can still write into its shared memory
+  // no CTA may leave while a peer can still write into its shared memory;
+  // the tensor memory is released once every warp is done with it
   __syncwarp();
+  tmem_fence_before();
   cluster_sync_all();
+  tmem_fence_after();
+  if (warp == 0) tmem_dealloc512(sh.tmem_base);
 }
 
 // ---- host side ------------------------------------------------------------------
 
+// The kernel takes all 512 TMEM columns, so no two of its CTAs may share an
+// SM (two clusters each waiting in tcgen05.alloc for the other could never
+// finish): every launch asks for more than half of an SM's shared memory.
+constexpr size_t kMinSmem = 116 * 1024;
+
 size_t shared_bytes(int U) {
   const size_t SU = size_t(U) * kConsumers * 8;  // padded slice, see the kernel
-  return ((sizeof(Shared) + 127) & ~size_t(127)) + kStages * SU * 2 + SU * 4;
+  const size_t b = ((sizeof(Shared) + 127) & ~size_t(127)) + kStages * SU * 2;
+  return b < kMinSmem ? kMinSmem : b;
 }
 
 constexpr size_t kSmemLimit = 227 * 1024;
