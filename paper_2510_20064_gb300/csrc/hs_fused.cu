@@ -7,26 +7,27 @@
 // cluster of C CTAs takes one (b,k) tile, each CTA a V/C slice, and loops
 // persistently over tiles:
 //   * the CTA's slice of every row of its tiles -- the target row, then the
-//     N drafter rows -- streams into a kStages-deep shared-memory ring with
-//     cp.async.bulk (TMA; each CTA reads its own slice, no multicast);
+//     N drafter rows -- streams into a 3-stage shared-memory ring with
+//     cp.async.bulk (TMA; each CTA reads its own slice, no multicast); a
+//     coordinator warp refills a stage as soon as every consumer has read it;
 //   * 15 consumer warps load a row from the ring into registers, form
 //     e_v = 2^{z_v c - o_w} with o_w = c * (the warp's max), c = log2e/T,
-//     and their sum (one ex2 per logit), and park the exponentials in
-//     tensor memory (TMEM), each thread in its own lane;
-//   * a coordinator warp merges the 15 warps' (offset, sum) pairs of a row,
-//     stores the CTA's pair into every peer CTA (distributed shared memory)
-//     and arrives on the peer's mbarrier, and refills the row's ring stage;
-//     every consumer thread then merges the C pairs into the row's offset O
-//     and normaliser Z, so p_v or q_v = e_v 2^{o_w - O} / Z;
-//   * the target's p goes to TMEM for the tile's N drafters; a drafter row
-//     adds sum_v min(p_v, q_v) to its per-warp partial;
-//   * the coordinator sums each tile's per-warp partials and sends them to
-//     the cluster's rank 0, whose coordinator sums them in rank order and
-//     writes alpha[:, b, k] one tile later.
-// Rows are software-pipelined three deep: pass 1 of row g+2 runs before
-// pass 2 of row g, so a row's exchange has two rows of work to hide behind.
-// Every wait is bounded; on expiry the kernel records HS_ERR_TIMEOUT and
-// finishes without waiting further.
+//     and their sum (one ex2 per logit, values kept in registers);
+//   * the cluster merges the per-CTA (offset, sum) pairs through distributed
+//     shared memory: every CTA stores its pair into each peer and arrives on
+//     the peer's mbarrier; then every thread knows the row's offset O and
+//     normaliser Z, and p_v or q_v = e_v 2^{o_t - O} / Z;
+//   * the target's p stays in shared memory (fp32) for the tile's N drafters;
+//     a drafter row adds sum_v min(p_v, q_v) to its per-warp partial;
+//   * at the end of a tile the coordinator sums the warps' N partials and
+//     sends them to the cluster's rank 0, whose coordinator sums them in rank
+//     order and writes alpha[:, b, k] one tile later.  The coordinator never
+//     blocks: its waits poll, servicing ring refills meanwhile, and no
+//     consumer warp waits for another warp of its CTA.
+// Rows are software-pipelined: the pass over row g+1's logits runs while
+// row g's cluster exchange is in flight, so each thread holds two rows of
+// exponentials (eA / eB).  Every wait is bounded; on expiry the kernel
+// records HS_ERR_TIMEOUT and finishes without waiting further.
 #include <math.h>
 #include <stdint.h>
 
@@ -37,9 +38,9 @@ namespace hs {
 namespace fused {
 namespace {
 
-// 15 consumer warps + 1 coordinator warp: 16 warps put 4 on each SM
-// sub-partition and 128 registers per thread; each consumer thread keeps
-// p and two rows of exponentials (3 x 8U columns) in TMEM.
+// 15 consumer warps + 1 load warp: 16 warps put 4 on each SM sub-partition,
+// which leaves 128 registers per thread for the two rows of exponentials a
+// consumer thread keeps.
 constexpr int kConsumerWarps = 15;
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;
@@ -587,8 +588,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
 
     // pass 2 of row g (exponentials in TMEM slot g & 1): target -> p into
     // TMEM; drafter i -> alpha partial
-    auto pass2 = [&](int g, float o, float o_used) {
-      const int j = g / R, r = g - (g / R) * R;
+    auto pass2 = [&](int g, int j, int r, float o, float o_used) {
       float O, invZ;
       const bool ok = gather(g, O, invZ);
       const float f = (o == -INFINITY || !ok) ? 0.f : ex2(o_used - O) * invZ;
@@ -667,11 +667,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     // so the cluster exchange of a row has two rows of work to hide behind
     f2_t E[U * 4];
     float o0 = 0.f, ou0 = 0.f, o1 = 0.f, ou1 = 0.f;  // offsets of rows in slots 0, 1
+    int jj = 0, rr = 0;
     for (int g = -2; g < G; ++g) {
       const bool more = g + 2 < G;
       float on = 0.f, oun = 0.f;
       if (more) pass1(g + 2, E, on, oun);
-      if (g >= 0) pass2(g, (g & 1) ? o1 : o0, (g & 1) ? ou1 : ou0);
+      if (g >= 0) {
+        pass2(g, jj, rr, (g & 1) ? o1 : o0, (g & 1) ? ou1 : ou0);
+        if (++rr == R) { rr = 0; ++jj; }
+      }
       if (more) {
         store_row(g & 1, E);
         if (g & 1) {
