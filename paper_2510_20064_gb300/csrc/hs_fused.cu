@@ -46,6 +46,7 @@ constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;
 constexpr int kStages = 4;
 constexpr int kXSlots = 8;  // rows whose exchange may be in flight at once
+constexpr int kXArm = 4;    // the xbar phase of row g + kXArm is armed at row g
 constexpr int kASlots = 8;  // tiles whose alpha partials may be in flight (rank 0)
 constexpr int kTSlots = 4;  // tiles whose per-warp partials await the coordinator
 constexpr int kMaxU = 5;    // 16-byte vectors per consumer thread and row
@@ -62,8 +63,10 @@ struct __align__(16) Shared {
   float2 red[kXSlots][16];                // per-warp (offset, sum) of a row
   float2 xch[kXSlots][kMaxC];             // per-rank (offset, sum) of a row
   float acc[kTSlots][kMaxN][kConsumerWarps];  // per-warp alpha partials of a tile
-  uint32_t tvalid[kTSlots];               // the tile's target row is usable
-  uint32_t dvalid[kTSlots];               // bit i: drafter i's row is usable
+  uint64_t rowbar[kXSlots];               // a row's per-warp scales are published
+  float rowf[kXSlots][16];                // per-warp scale f: p or q = f * exponential
+  uint32_t tval[kASlots];                 // tile's target row is usable
+  uint32_t dval[kASlots];                 // bit i: tile's drafter i row is usable
   float clacc[kASlots][kMaxC][kMaxN];     // per-rank alpha partials (rank 0)
   int error;
   uint32_t tmem_base;  // tensor memory: p and two rows of exponentials per thread
@@ -123,6 +126,14 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
 }
 // try_wait suspends the thread until the phase completes or about 1 ms has
 // passed, so a waiting warp does not spin through the issue slots.
+__device__ __forceinline__ bool mbar_test_cta(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n\t.reg .pred p;\n\t"
+               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+               "selp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(ok) : "r"(bar), "r"(parity), "r"(1000000u) : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile("{\n\t.reg .pred p;\n\t"
@@ -137,17 +148,15 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
                "[%0], [%1], %2, [%3];"
                :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
-// Arrive on a barrier in another CTA of the cluster, ordering this thread's
-// earlier shared::cluster stores before the arrival.
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];"
-               :: "r"(cluster_bar) : "memory");
+// Store a pair into another CTA of the cluster; the store itself completes 8
+// bytes of the transaction count of that CTA's mbarrier (no fence needed).
+__device__ __forceinline__ void st_async_f2(uint32_t a, float x, float y, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];"
+               :: "r"(a), "f"(x), "f"(y), "r"(bar) : "memory");
 }
-__device__ __forceinline__ void st_cluster_f2(uint32_t a, float x, float y) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" :: "r"(a), "f"(x), "f"(y) : "memory");
-}
-__device__ __forceinline__ void st_cluster_f(uint32_t a, float x) {
-  asm volatile("st.shared::cluster.f32 [%0], %1;" :: "r"(a), "f"(x) : "memory");
+__device__ __forceinline__ void st_async_f(uint32_t a, float x, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];"
+               :: "r"(a), "f"(x), "r"(bar) : "memory");
 }
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
   uint4 v;
@@ -179,6 +188,13 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, Shared
                                            int* dev_status, bool fast_fail = true) {
   if (mbar_test(bar, parity)) return true;
   return wait_slow(bar, parity, sh, dev_status, fast_fail);
+}
+// The same for a barrier that only this CTA's own threads complete: the
+// fast path acquires at CTA scope.
+__device__ __forceinline__ bool wait_local(uint32_t bar, uint32_t parity, Shared& sh,
+                                           int* dev_status) {
+  if (mbar_test_cta(bar, parity)) return true;
+  return wait_slow(bar, parity, sh, dev_status, true);
 }
 
 // ---- per-element helpers ----------------------------------------------------
@@ -287,19 +303,6 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, f2_t* v) {
   for (int i = 0; i < NV; ++i) v[i] = pk(f[2 * i], f[2 * i + 1]);
 }
 
-// Order-preserving int key of a float (NaN above +inf), so that a warp's
-// maximum is one redux.sync.
-__device__ __forceinline__ int fkey(float f) {
-  const int b = __float_as_int(f);
-  return (f != f) ? 0x7fffffff : (b >= 0 ? b : b ^ 0x7fffffff);
-}
-__device__ __forceinline__ float kfloat(int k) {
-  return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff);  // 0x7fffffff is a NaN
-}
-__device__ __forceinline__ float warp_max_key(float f) {
-  return kfloat(__reduce_max_sync(0xffffffffu, fkey(f)));
-}
-
 // Warp maximum, NaN if any lane holds a NaN (sm_100+ redux on f32).
 __device__ __forceinline__ float warp_max_f(float f) {
   float r;
@@ -310,20 +313,6 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
   float r;
   asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
   return r;
-}
-__device__ __forceinline__ float rcp_approx(float x) {
-  float r;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
-  return r;
-}
-// Merge (offset o, sum s) pairs held by the lanes of a warp: the largest
-// offset O (NaN wins, -inf means "no finite logit") and sum_l s_l 2^{o_l - O}.
-__device__ __forceinline__ void warp_merge(float& o, float& s) {
-  const float O = warp_max_key(o);
-  float t = (o == -INFINITY || O == -INFINITY) ? 0.f : s * ex2(o - O);
-  t = warp_sum(t);
-  o = O;
-  s = t;
 }
 
 // ---- the kernel ---------------------------------------------------------------
@@ -418,11 +407,20 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     for (int s = 0; s < kStages; ++s) mbar_init(saddr(&sh.full[s]), 1);
     for (int x = 0; x < kXSlots; ++x) {
       mbar_init(saddr(&sh.redbar[x]), kConsumerWarps);
-      mbar_init(saddr(&sh.xbar[x]), C);
+      mbar_init(saddr(&sh.xbar[x]), 1);
+      mbar_init(saddr(&sh.rowbar[x]), 1);
     }
     for (int a = 0; a < kTSlots; ++a) mbar_init(saddr(&sh.accbar[a]), kConsumerWarps);
-    for (int a = 0; a < kASlots; ++a) mbar_init(saddr(&sh.abar[a]), C * N);
+    for (int a = 0; a < kASlots; ++a) mbar_init(saddr(&sh.abar[a]), 1);
     sh.error = 0;
+    // each row's xbar phase: one local arrival (the arm) plus 8 bytes from
+    // every rank; the first kXArm rows are armed before any rank can send
+    for (int g = 0; g < kXArm && g < G; ++g) mbar_arrive_tx(saddr(&sh.xbar[g]), 8u * C);
+    // rank 0's abar phase of tile j: one local arrival (the arm) plus 4 bytes
+    // per drafter from every rank; tiles 0..kASlots-1 are armed here, tile
+    // j + kASlots once tile j is finished
+    for (int a = 0; a < kASlots && a < my_tiles; ++a)
+      mbar_arrive_tx(saddr(&sh.abar[a]), 4u * N * C);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) tmem_alloc512(saddr(&sh.tmem_base));
@@ -453,13 +451,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
         float t = 0.f;
         for (uint32_t rr = 0; rr < C; ++rr) t += sh.clacc[j % kASlots][rr][lane];
         const bool bad_path = p.path && (p.path[tile] < 0 || p.path[tile] >= p.M);
-        const int ts = j % kTSlots;
-        if (bad_path || !sh.tvalid[ts] || !((sh.dvalid[ts] >> lane) & 1u)) {
+        if (bad_path || !sh.tval[j % kASlots] || !((sh.dval[j % kASlots] >> lane) & 1u)) {
           t = __int_as_float(0x7fc00000);
           report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
         }
         p.alpha[(int64_t(lane) * B + b) * P + k] = t;
       }
+      __syncwarp();
+      if (lane == 0 && j + kASlots < my_tiles)
+        mbar_arrive_tx(saddr(&sh.abar[j % kASlots]), 4u * N * C);
     };
     auto reduce_tile = [&](int j) {  // tile j's partials -> rank 0
       const int ts = j % kTSlots;
@@ -467,10 +467,51 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       if (lane < N) {
         float t = 0.f;
         for (int w = 0; w < kConsumerWarps; ++w) t += sh.acc[ts][lane][w];
-        st_cluster_f(mapa(saddr(&sh.clacc[j % kASlots][rank][lane]), 0), t);
-        mbar_arrive_remote(mapa(saddr(&sh.abar[j % kASlots]), 0));
+        st_async_f(mapa(saddr(&sh.clacc[j % kASlots][rank][lane]), 0), t,
+                   mapa(saddr(&sh.abar[j % kASlots]), 0));
       }
       if (rank == 0 && j > 0) finish(j - 1);  // long since complete
+    };
+    // B(g): every rank's pair of row g -> the row's offset O and normaliser
+    // Z (a butterfly over each group of 8 lanes, lane l holding rank l & 7),
+    // then each consumer warp's scale f_w = 2^{o_w - O} / Z and the row's
+    // validity; published through rowbar.
+    int rB = 0, jB = 0;  // row within tile and tile of the next B step
+    auto publish = [&](int g) {
+      const int x = g % kXSlots;
+      wait_phase(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
+      // every lane merges the C pairs itself, in rank order
+      float2 v[kMaxC];
+#pragma unroll
+      for (int rr = 0; rr < kMaxC; ++rr)
+        v[rr] = rr < int(C) ? sh.xch[x][rr] : make_float2(-INFINITY, 0.f);
+      float O = v[0].x;
+#pragma unroll
+      for (int rr = 1; rr < kMaxC; ++rr) O = fmax_nan(O, v[rr].x);
+      float Z = 0.f;
+#pragma unroll
+      for (int rr = 0; rr < kMaxC; ++rr)
+        Z += (v[rr].x == -INFINITY || O == -INFINITY) ? 0.f : v[rr].y * ex2(v[rr].x - O);
+      const bool valid = isfinite(O) && Z > 0.f;
+      if (lane < kConsumerWarps) {
+        const float o = sh.red[x][lane].x;  // the offset warp `lane` used
+        sh.rowf[x][lane] = (!valid || o == -INFINITY) ? 0.f : ex2(o - O) / Z;
+      }
+      if (lane == 0) {
+        const int a = jB % kASlots;
+        if (rB == 0) {
+          sh.tval[a] = valid ? 1u : 0u;
+          sh.dval[a] = 0u;
+        } else if (valid) {
+          sh.dval[a] |= 1u << (rB - 1);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(saddr(&sh.rowbar[x]));
+      if (++rB == R) {
+        rB = 0;
+        ++jB;
+      }
     };
     int reduced = 0;  // tiles sent to rank 0
     for (int g = 0; g < G; ++g) {
@@ -479,15 +520,22 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       if (lane == 0 && g + kStages < G)
         issue(sh, ring + (g % kStages) * stage_bytes, g + kStages, walk.next(p, ncl, slice0),
               bytes);
-      float2 v = lane < kConsumerWarps ? sh.red[x][lane] : make_float2(-INFINITY, 0.f);
-      float oc = v.x, sc = v.y;
-      warp_merge(oc, sc);
-      if (lane < int(C)) {
-        st_cluster_f2(mapa(saddr(&sh.xch[x][rank]), lane), oc, sc);
-        mbar_arrive_remote(mapa(saddr(&sh.xbar[x]), lane));
-      }
+      // row g - kXArm's exchange is complete here (the consumers have passed
+      // pass 2 of row g - 3), so its slot can be armed for row g + kXArm,
+      // which no rank sends before this CTA has posted row g + 1
+      if (lane == 0 && g + kXArm < G)
+        mbar_arrive_tx(saddr(&sh.xbar[(g + kXArm) % kXSlots]), 8u * C);
+      const float2 v = lane < kConsumerWarps ? sh.red[x][lane] : make_float2(-INFINITY, 0.f);
+      const float oc = warp_max_f(v.x);
+      float sc = (v.x == -INFINITY || oc == -INFINITY) ? 0.f : v.y * ex2(v.x - oc);
+#pragma unroll
+      for (int d = 8; d > 0; d >>= 1) sc += __shfl_xor_sync(0xffffffffu, sc, d);
+      if (lane < int(C))
+        st_async_f2(mapa(saddr(&sh.xch[x][rank]), lane), oc, sc, mapa(saddr(&sh.xbar[x]), lane));
+      if (g > 0) publish(g - 1);
       while (reduced < my_tiles && (reduced + 1) * R + 2 <= g) reduce_tile(reduced++);
     }
+    if (G > 0) publish(G - 1);
     while (reduced < my_tiles) reduce_tile(reduced++);
     if (G > 0 && rank == 0) finish(my_tiles - 1);
     // drain: every copy has landed before the CTA may exit
@@ -498,7 +546,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   } else if (G > 0) {
     // ------------------------------ consumers -----------------------------
     const float c = p.c;
-    uint32_t tvalid = 0, dvalid = 0;  // target row usable; bit i: drafter i usable
     // the last vector round holds the slice's tail: warps whose vectors there
     // all lie past the slice skip it (they would only see the -inf padding)
     const bool tail = (U - 1) * kConsumers + warp * 32 < len / 8;
@@ -510,9 +557,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     // pass 1: load row g from the ring (then release the stage); warp max;
     // exponentials relative to the warp's offset; post the warp's (offset,
     // sum) for the coordinator.  E keeps the exponentials (packed pairs).
-    auto pass1 = [&](int g, f2_t (&E)[U * 4], float& o, float& o_used) {
+    auto pass1 = [&](int g, f2_t (&E)[U * 4]) {
       const int s = g % kStages;
-      wait_phase(saddr(&sh.full[s]), uint32_t(g / kStages) & 1u, sh, p.dev_status);
+      wait_local(saddr(&sh.full[s]), uint32_t(g / kStages) & 1u, sh, p.dev_status);
       const uint32_t stage = saddr(ring + s * stage_bytes);
       uint32_t w[U * 4];
 #pragma unroll
@@ -530,8 +577,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
 #pragma unroll
         for (int q = 0; q + d < U * 2; q += 2 * d) mx[q] = pmax<DT>(mx[q], mx[q + d]);
       const float m = warp_max_f(fmax_nan(lo<DT>(mx[0]), hi<DT>(mx[0])));
-      o = (m == -INFINITY) ? -INFINITY : m * c;
-      o_used = (m == -INFINITY) ? 0.f : o;
+      const float o = (m == -INFINITY) ? -INFINITY : m * c;
+      const float o_used = (m == -INFINITY) ? 0.f : o;
       const f2_t cc = pk(c, c), off = pk(-o_used, -o_used);
       f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
@@ -567,37 +614,16 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       }
     };
 
-    // all ranks' pairs of row g: the row's offset O and 1/Z.  Lane l holds
-    // rank (l & 7)'s pair (neutral past C); a butterfly over each group of 8
-    // lanes leaves the same merged pair in every lane.
-    auto gather = [&](int g, float& O, float& invZ) -> bool {
-      const int x = g % kXSlots;
-      wait_phase(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
-      const int r8 = lane & 7;
-      const float2 v = r8 < int(C) ? sh.xch[x][r8] : make_float2(-INFINITY, 0.f);
-      float o = v.x;
-#pragma unroll
-      for (int d = 1; d < 8; d *= 2) o = fmax_nan(o, __shfl_xor_sync(0xffffffffu, o, d));
-      float t = (v.x == -INFINITY || o == -INFINITY) ? 0.f : v.y * ex2(v.x - o);
-#pragma unroll
-      for (int d = 1; d < 8; d *= 2) t += __shfl_xor_sync(0xffffffffu, t, d);
-      O = o;
-      invZ = rcp_approx(t);
-      return isfinite(o) && t > 0.f;
-    };
-
     // pass 2 of row g (exponentials in TMEM slot g & 1): target -> p into
     // TMEM; drafter i -> alpha partial
-    auto pass2 = [&](int g, int j, int r, float o, float o_used) {
-      float O, invZ;
-      const bool ok = gather(g, O, invZ);
-      const float f = (o == -INFINITY || !ok) ? 0.f : ex2(o_used - O) * invZ;
+    auto pass2 = [&](int g, int j, int r) {
+      const int x = g % kXSlots;
+      wait_local(saddr(&sh.rowbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
+      const float f = sh.rowf[x][warp];
       const f2_t ff = pk(f, f);
       const uint32_t te = tbase + uint32_t((1 + (g & 1)) * U * 8);
       tmem_wait_st();  // this row's exponentials and the tile's p have landed
       if (r == 0) {
-        tvalid = ok ? 1u : 0u;
-        dvalid = 0;
 #pragma unroll
         for (int u = 0; u < U; u += 2) {
           f2_t e[8];
@@ -618,7 +644,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
         return;
       }
       const int i = r - 1;
-      if (ok) dvalid |= 1u << i;
       f2_t acc[2] = {pk(0.f, 0.f), pk(0.f, 0.f)};
 #pragma unroll
       for (int u = 0; u < U; u += 2) {
@@ -653,39 +678,25 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       if (lane == 0) {
         const int ts = j % kTSlots;
         sh.acc[ts][i][warp] = a;
-        if (i == N - 1) {  // tile end: hand the partials to the coordinator
-          if (warp == 0) {
-            sh.tvalid[ts] = tvalid;
-            sh.dvalid[ts] = dvalid;
-          }
-          mbar_arrive(saddr(&sh.accbar[ts]));
-        }
+        if (i == N - 1) mbar_arrive(saddr(&sh.accbar[ts]));  // tile end
       }
     };
 
     // three rows in flight: pass 1 of row g+2 runs before pass 2 of row g,
     // so the cluster exchange of a row has two rows of work to hide behind
     f2_t E[U * 4];
-    float o0 = 0.f, ou0 = 0.f, o1 = 0.f, ou1 = 0.f;  // offsets of rows in slots 0, 1
-    int jj = 0, rr = 0;
+    int jj = 0, rr = 0;  // tile and row within tile of row g
     for (int g = -2; g < G; ++g) {
       const bool more = g + 2 < G;
-      float on = 0.f, oun = 0.f;
-      if (more) pass1(g + 2, E, on, oun);
+      if (more) pass1(g + 2, E);
       if (g >= 0) {
-        pass2(g, jj, rr, (g & 1) ? o1 : o0, (g & 1) ? ou1 : ou0);
-        if (++rr == R) { rr = 0; ++jj; }
-      }
-      if (more) {
-        store_row(g & 1, E);
-        if (g & 1) {
-          o1 = on;
-          ou1 = oun;
-        } else {
-          o0 = on;
-          ou0 = oun;
+        pass2(g, jj, rr);
+        if (++rr == R) {
+          rr = 0;
+          ++jj;
         }
       }
+      if (more) store_row(g & 1, E);
     }
   }
   // no CTA may leave while a peer can still write into its shared memory;
