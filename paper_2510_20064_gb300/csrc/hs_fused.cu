@@ -303,6 +303,11 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, f2_t* v) {
   for (int i = 0; i < NV; ++i) v[i] = pk(f[2 * i], f[2 * i + 1]);
 }
 
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
 // Warp maximum, NaN if any lane holds a NaN (sm_100+ redux on f32).
 __device__ __forceinline__ float warp_max_f(float f) {
   float r;
@@ -444,7 +449,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
         issue(sh, ring + g * stage_bytes, g, walk.next(p, ncl, slice0), bytes);
     }
     auto finish = [&](int j) {  // rank 0: alpha[:, b, k] of tile j
-      wait_phase(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u, sh, p.dev_status);
+      wait_local(saddr(&sh.abar[j % kASlots]), uint32_t(j / kASlots) & 1u, sh, p.dev_status);
       if (lane < N) {
         const int64_t tile = int64_t(cid) + int64_t(j) * ncl;
         const int64_t b = tile / P, k = tile % P;
@@ -463,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     };
     auto reduce_tile = [&](int j) {  // tile j's partials -> rank 0
       const int ts = j % kTSlots;
-      wait_phase(saddr(&sh.accbar[ts]), uint32_t(j / kTSlots) & 1u, sh, p.dev_status);
+      wait_local(saddr(&sh.accbar[ts]), uint32_t(j / kTSlots) & 1u, sh, p.dev_status);
       if (lane < N) {
         float t = 0.f;
         for (int w = 0; w < kConsumerWarps; ++w) t += sh.acc[ts][lane][w];
@@ -479,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     int rB = 0, jB = 0;  // row within tile and tile of the next B step
     auto publish = [&](int g) {
       const int x = g % kXSlots;
-      wait_phase(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
+      wait_local(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
       // every lane merges the C pairs itself, in rank order
       float2 v[kMaxC];
 #pragma unroll
@@ -495,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       const bool valid = isfinite(O) && Z > 0.f;
       if (lane < kConsumerWarps) {
         const float o = sh.red[x][lane].x;  // the offset warp `lane` used
-        sh.rowf[x][lane] = (!valid || o == -INFINITY) ? 0.f : ex2(o - O) / Z;
+        sh.rowf[x][lane] = (!valid || o == -INFINITY) ? 0.f : ex2(o - O) * rcp_approx(Z);
       }
       if (lane == 0) {
         const int a = jB % kASlots;
@@ -516,7 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     int reduced = 0;  // tiles sent to rank 0
     for (int g = 0; g < G; ++g) {
       const int x = g % kXSlots;
-      wait_phase(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
+      wait_local(saddr(&sh.redbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
       if (lane == 0 && g + kStages < G)
         issue(sh, ring + (g % kStages) * stage_bytes, g + kStages, walk.next(p, ncl, slice0),
               bytes);
