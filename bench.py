@@ -133,10 +133,20 @@ def measured_hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
+# the sources of the kernels a feedback call of each mode launches
+KERNEL_SOURCES = {
+    "stochastic": ("hs_common.cuh", "hs_feedback.cu", "hs_fused.cu", "hs_fused.h",
+                   "hs_stream.cu", "hs_stream.h"),
+    "greedy": ("hs_common.cuh", "hs_feedback.cu", "hs_greedy.cu", "hs_greedy.h"),
+}
+
+
+def kernel_source_hash(mode: str) -> str:
+    """Hash of the kernel sources a feedback call of `mode` runs: a committed
+    ncu summary counts only while the kernels it measured are unchanged."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2510_20064_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in KERNEL_SOURCES[mode]:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
@@ -154,7 +164,7 @@ def profiled_traffic(workload: str, mode: str):
             if ":" in line and line.strip().startswith("- "):
                 k, v = line.strip()[2:].split(":", 1)
                 fields[k.strip()] = v.strip().strip("`")
-    if fields.get("kernel_source_hash") != kernel_source_hash():
+    if fields.get("kernel_source_hash") != kernel_source_hash(mode):
         return None
     try:
         return int(fields["dram_bytes_per_call"])
