@@ -385,6 +385,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   // past the CTA's slice is -inf (set once, below)
   constexpr int SU = U * kConsumers * 8;
   constexpr uint32_t stage_bytes = SU * 2;
+  // TMEM: the consumer warps of one lane quadrant (warps w, w+4, ...) each
+  // take 3 * 8U columns (p and two row slots) of the 512
+  static_assert(((kConsumerWarps + 3) / 4) * 3 * U * 8 <= 512, "TMEM columns");
   unsigned char* ring = smem_raw + ((sizeof(Shared) + 127) & ~size_t(127));
 
   const int tid = threadIdx.x;
