@@ -11,6 +11,34 @@ namespace hs {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// ---- programmatic dependent launch ------------------------------------------
+// Every kernel here is launched with programmatic stream serialization, so
+// that it can be scheduled while the previous kernel of the stream finishes.
+// pdl_wait() blocks until that kernel has completed and its memory is
+// visible: each kernel calls it before touching global memory another
+// kernel may write or read.  pdl_trigger() lets the next kernel be scheduled
+// early.  Both are no-ops in a launch without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---- element decode -------------------------------------------------------
 // bf16 is the upper half of a binary32, so widening is a shift (exact);
 // fp16 widens with the hardware conversion (exact); fp32 is read as is.

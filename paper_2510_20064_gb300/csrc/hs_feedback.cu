@@ -62,6 +62,7 @@ __global__ void __launch_bounds__(kThreads) row_stats_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int B, int P, int V, float c,
     RowStat* __restrict__ stats) {
+  pdl_wait();
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kChunk = kThreads * kUnroll * kV;
   __shared__ float red_m[kWarps];
@@ -123,6 +124,7 @@ __global__ void __launch_bounds__(kThreads) row_stats_kernel(
     st.argmax = valid ? ra : (bad_path ? -2 : -1);
     stats[r] = st;
   }
+  pdl_trigger();
 }
 
 template <int DT, bool VEC>
@@ -130,6 +132,7 @@ __global__ void __launch_bounds__(kThreads) overlap_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int N, int B, int P, int V, float c,
     const RowStat* __restrict__ stats, float* __restrict__ partial, int nchunk) {
+  pdl_wait();
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kS = kUnroll * kV;
   constexpr int kChunk = kThreads * kS;
@@ -167,6 +170,7 @@ __global__ void __launch_bounds__(kThreads) overlap_kernel(
     for (int ww = 0; ww < kWarps; ++ww) s += red[ww * N + i];
     partial[(tile * nchunk + j) * N + i] = s;
   }
+  pdl_trigger();
 }
 
 // One warp per (i, b): lanes sum the chunk partials of a position in a fixed
@@ -175,6 +179,7 @@ __global__ void finalize_kernel(const RowStat* __restrict__ stats,
                                 const float* __restrict__ partial, int nchunk, int N,
                                 int B, int P, float* __restrict__ alpha,
                                 float* __restrict__ e_len, int* dev_status) {
+  pdl_wait();
   const int64_t gw = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   if (gw >= int64_t(N) * B) return;  // whole warp
   const int l = threadIdx.x & 31;
@@ -255,16 +260,19 @@ hs_status launch_two_pass(const void* target, const int32_t* path, int M, const 
   RowStat* stats = reinterpret_cast<RowStat*>(static_cast<char*>(ws) + L.stats_off);
   float* partial = reinterpret_cast<float*>(static_cast<char*>(ws) + L.partial_off);
   const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
-  row_stats_kernel<DT, VEC><<<rows, kThreads, 0, stream>>>(target, path, M, drafter, B, P, V, c,
-                                                           stats);
+  if (launch_pdl(row_stats_kernel<DT, VEC>, dim3(rows), dim3(kThreads), 0, stream, target, path,
+                 M, drafter, B, P, V, c, stats) != cudaSuccess)
+    return HS_ERR_CUDA;
   const size_t smem = size_t(kWarps) * N * sizeof(float);
   dim3 grid(unsigned(int64_t(B) * P), unsigned(L.nchunk));
-  overlap_kernel<DT, VEC><<<grid, kThreads, smem, stream>>>(target, path, M, drafter, N, B, P, V,
-                                                           c, stats, partial, L.nchunk);
+  if (launch_pdl(overlap_kernel<DT, VEC>, grid, dim3(kThreads), smem, stream, target, path, M,
+                 drafter, N, B, P, V, c, stats, partial, L.nchunk) != cudaSuccess)
+    return HS_ERR_CUDA;
   const int64_t threads = int64_t(N) * B * 32;
-  finalize_kernel<<<unsigned((threads + 255) / 256), 256, 0, stream>>>(
-      stats, partial, L.nchunk, N, B, P, alpha, e_len, dev_status);
-  return cudaGetLastError() == cudaSuccess ? HS_OK : HS_ERR_CUDA;
+  if (launch_pdl(finalize_kernel, dim3(unsigned((threads + 255) / 256)), dim3(256), 0, stream,
+                 stats, partial, L.nchunk, N, B, P, alpha, e_len, dev_status) != cudaSuccess)
+    return HS_ERR_CUDA;
+  return HS_OK;
 }
 
 template <int DT>

@@ -390,6 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   static_assert(((kConsumerWarps + 3) / 4) * 3 * U * 8 <= 512, "TMEM columns");
   unsigned char* ring = smem_raw + ((sizeof(Shared) + 127) & ~size_t(127));
 
+  pdl_trigger();  // the small e_len kernel may take the SMs no cluster uses
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_rank();
@@ -435,6 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   tmem_fence_before();
   cluster_sync_all();
   tmem_fence_after();
+  pdl_wait();  // the set-up above overlaps the previous kernel of the stream
 
   if (warp == kConsumerWarps) {
     // ---------------------------- coordinator -----------------------------
@@ -762,11 +764,13 @@ hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
     configured_smem = int(smem);
   }
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = pl.C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
@@ -786,6 +790,7 @@ hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
   }
   const int nclusters = max(1, min(p.ntiles, max_clusters));
   cfg.gridDim = dim3(unsigned(nclusters * pl.C));
+  cfg.numAttrs = 2;  // cluster shape + programmatic dependent launch
   if (cudaLaunchKernelEx(&cfg, kern, p) != cudaSuccess) return HS_ERR_CUDA;
   return HS_OK;
 }
@@ -803,6 +808,7 @@ hs_status launch_dt(const Params& p, const Plan& pl, cudaStream_t s) {
 
 __global__ void elen_kernel(const float* __restrict__ alpha, int64_t NB, int P,
                             float* __restrict__ e_len) {
+  pdl_wait();
   const int64_t idx = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (idx >= NB) return;
   const float* a = alpha + idx * P;
@@ -851,8 +857,9 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   if (st != HS_OK) return st;
   if (e_len) {
     const int64_t nb = int64_t(N) * B;
-    elen_kernel<<<unsigned((nb + 255) / 256), 256, 0, stream>>>(alpha, nb, P, e_len);
-    if (cudaGetLastError() != cudaSuccess) return HS_ERR_CUDA;
+    if (launch_pdl(elen_kernel, dim3(unsigned((nb + 255) / 256)), dim3(256), 0, stream, alpha,
+                   nb, P, e_len) != cudaSuccess)
+      return HS_ERR_CUDA;
   }
   return HS_OK;
 }

@@ -36,6 +36,7 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int B, int P, int V, Part* __restrict__ parts,
     int nchunk) {
+  pdl_wait();
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kS = kUnroll * kV;
   __shared__ float red_m[kWarps];
@@ -77,6 +78,7 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
       if (red_m[q] == bm && red_a[q] < ba) ba = red_a[q];
     parts[r * nchunk + j] = Part{bm, ba};
   }
+  pdl_trigger();
 }
 
 // Row argmax from its chunk partials, by one warp: (max, first index).
@@ -100,6 +102,7 @@ __global__ void greedy_finalize_kernel(const Part* __restrict__ parts, int nchun
                                        const int32_t* __restrict__ path, int M, int N, int B,
                                        int P, float* __restrict__ alpha,
                                        float* __restrict__ e_len, int* dev_status) {
+  pdl_wait();
   const int64_t gw = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   if (gw >= int64_t(N) * B) return;  // whole warp
   const int64_t i = gw / B, b = gw % B;
@@ -141,12 +144,14 @@ hs_status launch_t(const void* target, const int32_t* path, int M, const void* d
   Part* parts = static_cast<Part*>(ws);
   const int nchunk = int((V + chunk_of<DT>() - 1) / chunk_of<DT>());
   const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
-  argmax_chunk_kernel<DT, VEC><<<dim3(rows, unsigned(nchunk)), kThreads, 0, s>>>(
-      target, path, M, drafter, B, P, V, parts, nchunk);
+  if (launch_pdl(argmax_chunk_kernel<DT, VEC>, dim3(rows, unsigned(nchunk)), dim3(kThreads), 0,
+                 s, target, path, M, drafter, B, P, V, parts, nchunk) != cudaSuccess)
+    return HS_ERR_CUDA;
   const int64_t threads = int64_t(N) * B * 32;
-  greedy_finalize_kernel<<<unsigned((threads + 255) / 256), 256, 0, s>>>(
-      parts, nchunk, path, M, N, B, P, alpha, e_len, dev_status);
-  return cudaGetLastError() == cudaSuccess ? HS_OK : HS_ERR_CUDA;
+  if (launch_pdl(greedy_finalize_kernel, dim3(unsigned((threads + 255) / 256)), dim3(256), 0, s,
+                 parts, nchunk, path, M, N, B, P, alpha, e_len, dev_status) != cudaSuccess)
+    return HS_ERR_CUDA;
+  return HS_OK;
 }
 
 template <int DT>

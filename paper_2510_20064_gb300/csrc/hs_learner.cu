@@ -56,6 +56,7 @@ __device__ __forceinline__ float warp_min(float v) {
 }
 
 __global__ void __launch_bounds__(kWarpsPerBlock * 32) learner_kernel(LearnerArgs a) {
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int64_t b = int64_t(blockIdx.x) * kWarpsPerBlock + (threadIdx.x >> 5);
   if (b >= a.B) return;  // whole warp leaves together
@@ -148,7 +149,9 @@ bool aligned4(const void* p) { return reinterpret_cast<uintptr_t>(p) % 4 == 0; }
 
 hs_status launch(const LearnerArgs& a, void* stream) {
   const unsigned blocks = unsigned((int64_t(a.B) + kWarpsPerBlock - 1) / kWarpsPerBlock);
-  learner_kernel<<<blocks, kWarpsPerBlock * 32, 0, static_cast<cudaStream_t>(stream)>>>(a);
+  if (launch_pdl(learner_kernel, dim3(blocks), dim3(kWarpsPerBlock * 32), 0,
+                 static_cast<cudaStream_t>(stream), a) != cudaSuccess)
+    return HS_ERR_CUDA;
   return cudaGetLastError() == cudaSuccess ? HS_OK : HS_ERR_CUDA;
 }
 

@@ -289,6 +289,7 @@ __device__ void overlap_item(const Params& p, Smem& sm, int y) {
 
 template <int DT>
 __global__ void __launch_bounds__(kThreads) stream_kernel(const Params p) {
+  pdl_wait();
   __shared__ Smem sm;
   const int G = gridDim.x;
   const int steps = (p.nitems + G - 1) / G + p.lag;
@@ -302,6 +303,7 @@ __global__ void __launch_bounds__(kThreads) stream_kernel(const Params p) {
 
 __global__ void elen_kernel(const float* __restrict__ alpha, int64_t NB, int P,
                             float* __restrict__ e_len) {
+  pdl_wait();
   const int64_t idx = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (idx >= NB) return;
   const float* a = alpha + idx * P;
@@ -411,8 +413,9 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   if (st != HS_OK) return st;
   if (e_len) {
     const int64_t nb = int64_t(N) * B;
-    elen_kernel<<<unsigned((nb + 255) / 256), 256, 0, stream>>>(alpha, nb, P, e_len);
-    if (cudaGetLastError() != cudaSuccess) return HS_ERR_CUDA;
+    if (launch_pdl(elen_kernel, dim3(unsigned((nb + 255) / 256)), dim3(256), 0, stream, alpha,
+                   nb, P, e_len) != cudaSuccess)
+      return HS_ERR_CUDA;
   }
   return HS_OK;
 }
