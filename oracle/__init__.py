@@ -49,6 +49,9 @@ def _bind(lib):
         "orc_loss_accept": ([P, I], D),
         "orc_feedback": ([P, P, I, I, I, I, I, D, I, P, P], I),
         "orc_feedback_path": ([P, P, I, P, I, I, I, I, I, D, I, P, P], I),
+        "orc_topl_set": ([P, I, I, I, P], None),
+        "orc_alpha_topl": ([P, P, I, I, D, I, I, P], I),
+        "orc_feedback_topl": ([P, P, I, P, I, I, I, I, I, D, I, I, P, P], I),
         "orc_hedge": ([P, I, D, P, P], None),
         "orc_normalhedge": ([P, P, P, I, P, P], I),
         "orc_learner_step": ([P, P, I, I, I, I, I, D, P, P, P, P, P], I),
@@ -167,6 +170,47 @@ class Oracle:
             st = self.lib.orc_feedback_path(_ptr(target), _ptr(path), M, _ptr(drafter),
                                             dtype_code(target), N, B, P, V, float(T),
                                             int(bool(greedy)), _ptr(alpha), _ptr(e_len))
+        return alpha, e_len, st
+
+    # ---- Thm 2: EAGLE tree with branching L ---------------------------------
+
+    def topl_set(self, row: np.ndarray, L: int) -> np.ndarray:
+        """Top_L(q) of one drafter row, in rank order (ties -> lower index)."""
+        row = np.ascontiguousarray(row)
+        L = min(int(L), row.shape[-1])
+        idx = np.empty(L, np.int32)
+        self.lib.orc_topl_set(_ptr(row), dtype_code(row), row.shape[-1], L, _ptr(idx))
+        return idx
+
+    def alpha_topl(self, zt: np.ndarray, zd: np.ndarray, T: float, greedy: bool, L: int):
+        zt = np.ascontiguousarray(zt)
+        zd = np.ascontiguousarray(zd)
+        a = ctypes.c_double()
+        st = self.lib.orc_alpha_topl(_ptr(zt), _ptr(zd), dtype_code(zt), zt.shape[-1], float(T),
+                                     int(bool(greedy)), int(L), ctypes.byref(a))
+        return a.value, st
+
+    def feedback_topl(self, target: np.ndarray, drafter: np.ndarray, T: float, greedy: bool,
+                      L: int, path: np.ndarray | None = None):
+        """As feedback() with Thm 2's acceptance: alpha = the target's mass
+        on the drafter's top-L tokens (greedy target: whether its argmax is
+        among them)."""
+        target = np.ascontiguousarray(target)
+        drafter = np.ascontiguousarray(drafter)
+        assert target.dtype == drafter.dtype
+        N, B, P, V = drafter.shape
+        alpha = np.empty((N, B, P), np.float64)
+        e_len = np.empty((N, B), np.float64)
+        if path is None:
+            assert target.shape == (B, P, V)
+            pp, M = None, 0
+        else:
+            pp = np.ascontiguousarray(path, dtype=np.int32)
+            M = target.shape[1]
+            assert target.shape == (B, M, V) and pp.shape == (B, P)
+        st = self.lib.orc_feedback_topl(_ptr(target), None if pp is None else _ptr(pp), M,
+                                        _ptr(drafter), dtype_code(target), N, B, P, V, float(T),
+                                        int(bool(greedy)), int(L), _ptr(alpha), _ptr(e_len))
         return alpha, e_len, st
 
     # ---- learners ----------------------------------------------------------

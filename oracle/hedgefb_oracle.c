@@ -12,6 +12,8 @@
  *   - Thm 1 (Sec. 2.2):      alpha = sum_x min(p(x), q(x)) = 1 - TV(p, q)
  *   - Thm 2 with L = 1 and a greedy target (Sec. 2.3): greedy alpha is the
  *                            indicator that the two argmaxes agree
+ *   - Thm 2 (Sec. 2.3), EAGLE tree with branching L: alpha is the target's
+ *                            mass on the drafter's top-L tokens
  *   - Thm 3 (Sec. 3.2):      counterfactual acceptance-length estimator
  *   - Sec. 3.3 / App. B.3:   length loss and acceptance-rate loss
  *   - App. B.1 remark:       Hedge, w_i <- w_i exp(-eta l_i), normalised
@@ -245,6 +247,100 @@ int orc_feedback_path(const void* tree, const int32_t* path, int M,
   if (M < 1 || !path) return ORC_BADARG;
   return feedback_impl(tree, path, M, drafter, dtype, N, B, P, V, T, greedy,
                        alpha, e_len);
+}
+
+/* ---- Thm 2: EAGLE draft tree with branching L -------------------------- */
+
+/* Top_L(q) of one drafter row: the L tokens the drafter ranks first.  The
+ * ranking is by the stored logit (softmax at any temperature keeps the
+ * order), larger first, ties toward the lower index; -inf logits rank last
+ * (their q is 0) and NaN never occurs here (unusable rows are rejected).
+ * Selection sort over the row, one pass per rank: plain and slow.  Writes
+ * idx[0..L-1] in rank order; L is at most V. */
+void orc_topl_set(const void* zd, int dtype, int V, int L, int* idx) {
+  for (int r = 0; r < L; ++r) {
+    int best = -1;
+    double bz = 0.0;
+    for (int v = 0; v < V; ++v) {
+      int taken = 0;
+      for (int q = 0; q < r; ++q)
+        if (idx[q] == v) { taken = 1; break; }
+      if (taken) continue;
+      double z = orc_decode(zd, dtype, v);
+      if (best < 0 || z > bz) { best = v; bz = z; }
+    }
+    idx[r] = best;
+  }
+}
+
+/* alpha for one (target row, drafter row) pair under Thm 2: the target's
+ * token is accepted iff it lies in the drafter's candidate set Top_L(q).
+ * Stochastic target: alpha = sum_{v in Top_L(q)} p(v).  Greedy target:
+ * alpha = 1[argmax p in Top_L(q)].  With L = 1 and a greedy target this is
+ * the argmax-agreement rule of the greedy mode. */
+int orc_alpha_topl(const void* zt, const void* zd, int dtype, int V, double T,
+                   int greedy, int L, double* alpha) {
+  if (L < 1) return ORC_BADARG;
+  if (L > V) L = V;
+  if (!row_ok(zd, dtype, V)) { *alpha = NAN; return ORC_NONFINITE; }
+  int* idx = (int*)malloc(sizeof(int) * (size_t)L);
+  orc_topl_set(zd, dtype, V, L, idx);
+  int st = ORC_OK;
+  if (greedy) {
+    int jt = orc_row_argmax(zt, dtype, V);
+    if (jt < 0) {
+      *alpha = NAN;
+      st = ORC_NONFINITE;
+    } else {
+      double a = 0.0;
+      for (int r = 0; r < L; ++r)
+        if (idx[r] == jt) a = 1.0;
+      *alpha = a;
+    }
+  } else {
+    double* Pt = (double*)malloc(sizeof(double) * (size_t)V);
+    st = orc_row_probs(zt, dtype, V, T, Pt);
+    double a = 0.0;
+    for (int r = 0; r < L; ++r) a += Pt[idx[r]];
+    *alpha = st ? NAN : a;
+    free(Pt);
+  }
+  free(idx);
+  return st;
+}
+
+/* A whole feedback call under Thm 2 (same layouts as orc_feedback /
+ * orc_feedback_path; path == NULL for a chain target). */
+int orc_feedback_topl(const void* target, const int32_t* path, int M,
+                      const void* drafter, int dtype, int N, int B, int P,
+                      int V, double T, int greedy, int L, double* alpha,
+                      double* e_len) {
+  if (N < 1 || B < 1 || P < 1 || V < 1 || L < 1 || (!greedy && !(T > 0.0)))
+    return ORC_BADARG;
+  if (path && M < 1) return ORC_BADARG;
+  size_t esz = (dtype == ORC_FP32) ? 4 : 2;
+  int status = ORC_OK;
+  for (int b = 0; b < B; ++b) {
+    for (int k = 0; k < P; ++k) {
+      if (path && (path[b * P + k] < 0 || path[b * P + k] >= M)) return ORC_BADARG;
+      int64_t row_t = (int64_t)b * P + k;               /* chain: target[b, k] */
+      if (path) row_t = (int64_t)b * M + path[b * P + k];  /* tree: its path row */
+      const char* zt = (const char*)target + (size_t)row_t * V * esz;
+      for (int i = 0; i < N; ++i) {
+        const int64_t row_d = ((int64_t)i * B + b) * P + k;  /* drafter[i, b, k] */
+        const char* zd = (const char*)drafter + (size_t)row_d * V * esz;
+        double a;
+        if (orc_alpha_topl(zt, zd, dtype, V, T, greedy, L, &a) != ORC_OK) status = ORC_NONFINITE;
+        alpha[row_d] = a;
+      }
+    }
+  }
+  for (int i = 0; i < N; ++i)
+    for (int b = 0; b < B; ++b) {
+      const double* gam = alpha + ((size_t)i * B + b) * P;  /* alpha_1..alpha_K */
+      e_len[i * B + b] = orc_elen_prefix(gam, P - 1);
+    }
+  return status;
 }
 
 /* ---- learners ---------------------------------------------------------- */

@@ -481,4 +481,131 @@ def check_learner_step_played_loss(o):
             assert np.allclose(w2.sum(axis=0), 1.0)
 
 
+# ---- Thm 2: EAGLE tree with branching L ----------------------------------------
+
+def topl_numpy(stored_row: np.ndarray, L: int) -> np.ndarray:
+    """The L tokens ranked first by stored logit, ties toward the lower index
+    (numpy lexsort: primary key -value, secondary key the index)."""
+    z = value(stored_row)
+    order = np.lexsort((np.arange(z.size), -z))
+    return order[:min(L, z.size)]
+
+
+def check_topl_set_lexsort(o):
+    """Top_L on tie-heavy rows (logits on a 1/4 grid, some -inf) equals the
+    lexsort ranking, for every L."""
+    rng = np.random.default_rng(41)
+    for kind in KINDS:
+        for V in (1, 5, 64, 300):
+            z = (rng.integers(-12, 12, V) / 4.0).astype(np.float32)
+            z[rng.random(V) < 0.1] = -np.inf
+            s = stored(z, kind)
+            for L in sorted({1, 2, 3, 7, 16, V}):
+                assert np.array_equal(o.topl_set(s, L), topl_numpy(s, L)), (kind, V, L)
+
+
+def check_topl_alpha_scipy(o):
+    """alpha = sum of scipy's softmax(z_t / T) over the drafter's top-L tokens."""
+    rng = np.random.default_rng(42)
+    for kind in KINDS:
+        for V in (2, 9, 100, 1000):
+            zt = stored(rng.normal(0, 3, V), kind)
+            zd = stored(value(zt) + rng.normal(0, 1.5, V), kind)
+            for T in (0.5, 1.0, 2.0):
+                p = probs(zt, T)
+                for L in (1, 3, 10):
+                    want = p[topl_numpy(zd, L)].sum()
+                    a, st = o.alpha_topl(zt, zd, T, False, L)
+                    assert st == orc.OK and abs(a - want) < 1e-12, (kind, V, T, L, a, want)
+
+
+def check_topl_special_cases(o):
+    """L = 1 under a greedy target is the argmax-agreement rule; L >= V puts
+    every token in the candidate set, so alpha = 1."""
+    rng = np.random.default_rng(43)
+    for kind in KINDS:
+        for trial in range(20):
+            V = int(rng.integers(2, 40))
+            zt = stored(rng.integers(-4, 4, V).astype(np.float32), kind)
+            zd = stored(rng.integers(-4, 4, V).astype(np.float32), kind)
+            a, st = o.alpha_topl(zt, zd, 1.0, True, 1)
+            want = 1.0 if np.argmax(value(zt)) == np.argmax(value(zd)) else 0.0
+            assert st == orc.OK and a == want
+            for greedy in (False, True):
+                a, st = o.alpha_topl(zt, zd, 0.8, greedy, V + int(rng.integers(0, 3)))
+                assert st == orc.OK and abs(a - 1.0) < 1e-12
+
+
+def check_topl_greedy_target_membership(o):
+    """Greedy target: alpha = 1 exactly when the target's argmax is among the
+    drafter's top-L tokens."""
+    rng = np.random.default_rng(44)
+    for trial in range(200):
+        V = int(rng.integers(3, 30))
+        L = int(rng.integers(1, V))
+        zt = rng.integers(-5, 5, V).astype(np.float32)
+        zd = rng.integers(-5, 5, V).astype(np.float32)
+        a, st = o.alpha_topl(zt, zd, 1.0, True, L)
+        want = 1.0 if np.argmax(zt) in set(topl_numpy(zd, L).tolist()) else 0.0
+        assert st == orc.OK and a == want, (V, L)
+
+
+def check_topl_mc_eagle(o):
+    """Monte Carlo of Thm 2 on V = 8: the target's sampled token is accepted
+    iff the drafter put it among its L children; the empirical rate matches
+    alpha within 5 sigma."""
+    rng = np.random.default_rng(45)
+    V, n = 8, 400_000
+    zt = rng.normal(0, 1.5, V).astype(np.float32)
+    zd = rng.normal(0, 1.5, V).astype(np.float32)
+    T = 0.9
+    p = probs(zt, T)
+    children = np.argsort(-zd, kind="stable")[:3]   # the drafter's 3 most likely tokens
+    x = rng.choice(V, size=n, p=p)
+    rate = np.isin(x, children).mean()
+    a, st = o.alpha_topl(zt, zd, T, False, 3)
+    sigma = math.sqrt(a * (1 - a) / n)
+    assert st == orc.OK and abs(rate - a) < 5 * sigma + 1e-12, (rate, a, sigma)
+
+
+def check_topl_nonfinite(o):
+    rng = np.random.default_rng(46)
+    zt = rng.normal(0, 1, 50).astype(np.float32)
+    zd = rng.normal(0, 1, 50).astype(np.float32)
+    bad = zd.copy()
+    bad[7] = np.nan
+    a, st = o.alpha_topl(zt, bad, 1.0, False, 4)
+    assert st == orc.NONFINITE and np.isnan(a)
+    badt = zt.copy()
+    badt[3] = np.inf
+    for greedy in (False, True):
+        a, st = o.alpha_topl(badt, zd, 1.0, greedy, 4)
+        assert st == orc.NONFINITE and np.isnan(a)
+
+
+def check_feedback_topl_layout(o):
+    """The whole-call layout: alpha[i,b,k] pairs target row (b,k) (or its path
+    row) with drafter row (i,b,k); e_len is 1 + sum of cumulative products of
+    alpha_1..alpha_K."""
+    rng = np.random.default_rng(47)
+    N, B, P, V, L, T = 3, 2, 4, 40, 5, 0.9
+    tgt = stored(rng.normal(0, 2, (B, P, V)), "bf16")
+    drf = stored(value(tgt)[None] + rng.normal(0, 1, (N, B, P, V)), "bf16")
+    M = 6
+    tree = stored(rng.normal(0, 2, (B, M, V)), "bf16")
+    path = rng.integers(0, M, (B, P)).astype(np.int32)
+    for use_path in (False, True):
+        a, e, st = o.feedback_topl(tree if use_path else tgt, drf, T, False, L,
+                                   path if use_path else None)
+        assert st == orc.OK
+        for i in range(N):
+            for b in range(B):
+                for k in range(P):
+                    zt = tree[b, path[b, k]] if use_path else tgt[b, k]
+                    want = probs(zt, T)[topl_numpy(drf[i, b, k], L)].sum()
+                    assert abs(a[i, b, k] - want) < 1e-12
+                want_e = 1.0 + np.cumprod(a[i, b, :P - 1]).sum()
+                assert abs(e[i, b] - want_e) < 1e-12
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -49,6 +49,21 @@ MUTANTS = {
     "greedy_inverted": ("a = (jt < 0 || jd < 0) ? NAN : (jt == jd ? 1.0 : 0.0);",
                         "a = (jt < 0 || jd < 0) ? NAN : (jt != jd ? 1.0 : 0.0);"),
     "played_loss_wrong_drafter": ("played[b] += f[selected[b]];", "played[b] += f[0];"),
+    "topl_ties_toward_higher_index": ("if (best < 0 || z > bz) { best = v; bz = z; }",
+                                      "if (best < 0 || z >= bz) { best = v; bz = z; }"),
+    "topl_smallest_first": ("if (best < 0 || z > bz) { best = v; bz = z; }",
+                            "if (best < 0 || z < bz) { best = v; bz = z; }"),
+    "topl_drops_last_candidate": ("for (int r = 0; r < L; ++r) a += Pt[idx[r]];",
+                                  "for (int r = 0; r + 1 < L; ++r) a += Pt[idx[r]];"),
+    "topl_greedy_first_child_only": ("for (int r = 0; r < L; ++r)\n        if (idx[r] == jt) a = 1.0;",
+                                     "for (int r = 0; r < 1; ++r)\n        if (idx[r] == jt) a = 1.0;"),
+    "topl_repeats_tokens": ("if (idx[q] == v) { taken = 1; break; }", "if (idx[q] == v) { break; }"),
+    "topl_target_index_transposed": ("int64_t row_t = (int64_t)b * P + k;",
+                                     "int64_t row_t = (int64_t)k * B + b;"),
+    "topl_drafter_index_transposed": ("const int64_t row_d = ((int64_t)i * B + b) * P + k;",
+                                      "const int64_t row_d = ((int64_t)b * N + i) * P + k;"),
+    "topl_elen_all_positions": ("e_len[i * B + b] = orc_elen_prefix(gam, P - 1);",
+                                "e_len[i * B + b] = orc_elen_prefix(gam, P);"),
     "hedge_state_not_cumulative": ("for (int i = 0; i < N; ++i) col[i] += f[i];",
                                    "for (int i = 0; i < N; ++i) col[i] = f[i];"),
 }
