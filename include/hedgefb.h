@@ -147,6 +147,45 @@ hs_status hs_feedback_path(const void* tree_target, const int32_t* path_idx,
                            size_t workspace_bytes, int* dev_status,
                            void* stream);
 
+/* Largest branching L the draft-tree entries accept. */
+#define HS_MAX_TREE_L 16
+
+/* Bytes of device workspace hs_feedback_topl / hs_feedback_topl_path need
+ * (one row statistic per target row); 0 for invalid sizes. */
+size_t hs_feedback_topl_workspace_size(int N, int B, int P, int V);
+
+/* Panoramic feedback for an EAGLE draft tree with branching L (Sec. 2.3,
+ * Thm 2): the drafter proposes its L most likely tokens as the children of
+ * a node, and the target's token is accepted iff it is one of them.  Same
+ * arguments and layouts as hs_feedback, plus
+ *   L          1 <= L <= HS_MAX_TREE_L: the drafter's candidate set is
+ *              Top_L(q_i), its L tokens with the largest stored logits
+ *              (the ranking of q does not depend on T), ties toward the
+ *              lower index, -inf logits last; L >= V takes every token.
+ *   greedy     0: alpha = sum_{v in Top_L(q_i)} p(v), p = softmax(z_target/T),
+ *                 fp32.  1: alpha = 1 if argmax p (stored logits, lowest
+ *                 index on ties) is in Top_L(q_i), else 0 -- exact.  With
+ *                 L = 1 this is hs_feedback's greedy rule.
+ *   workspace  device, hs_feedback_topl_workspace_size(...) bytes, 256-byte
+ *              aligned (required).
+ * The dynamic pruning of EAGLE-2 (Thm 2, last sentence) is not modelled:
+ * the candidate set is the plain top L.  Errors as in hs_feedback; a
+ * drafter row with NaN, +inf or no finite logit gives NaN and
+ * HS_ERR_NONFINITE. */
+hs_status hs_feedback_topl(const void* target, const void* drafter, int dtype, int N,
+                           int B, int P, int V, float temperature, int greedy, int L,
+                           float* alpha, float* e_len, void* workspace,
+                           size_t workspace_bytes, int* dev_status, void* stream);
+
+/* hs_feedback_topl with the target rows taken from a draft tree, as in
+ * hs_feedback_path (tree_target [B,M,V], path_idx [B,P] int32). */
+hs_status hs_feedback_topl_path(const void* tree_target, const int32_t* path_idx,
+                                int M, const void* drafter, int dtype, int N, int B,
+                                int P, int V, float temperature, int greedy, int L,
+                                float* alpha, float* e_len, void* workspace,
+                                size_t workspace_bytes, int* dev_status,
+                                void* stream);
+
 /* Hedge weights from cumulative losses (App. B.1 remark: w_i <- w_i
  * exp(-eta l_i) from w = 1, normalised, i.e. w = exp(-eta L) / Z).
  *   cum_loss  device, [N,B] fp32 cumulative loss L per (drafter, query).

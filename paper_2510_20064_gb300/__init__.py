@@ -23,6 +23,7 @@ HS_BF16, HS_FP16, HS_FP32 = 0, 1, 2
 HS_LOSS_LENGTH, HS_LOSS_ACCEPT = 0, 1
 HS_HEDGE, HS_NORMALHEDGE = 0, 1
 HS_MAX_LEARNER_N = 32
+HS_MAX_TREE_L = 16
 
 _DTYPES = {torch.bfloat16: HS_BF16, torch.float16: HS_FP16, torch.float32: HS_FP32}
 
@@ -36,6 +37,10 @@ SIGNATURES = {
     "hs_feedback": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_static": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _P], _I),
+    "hs_feedback_topl_workspace_size": ([_I, _I, _I, _I], _Z),
+    "hs_feedback_topl": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z, _P, _P], _I),
+    "hs_feedback_topl_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z,
+                               _P, _P], _I),
     "hs_hedge_update": ([_P, _I, _I, _F, _P, _P, _P], _I),
     "hs_normalhedge_update": ([_P, _P, _P, _I, _I, _P, _P], _I),
     "hs_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P], _I),
@@ -185,6 +190,54 @@ def hs_feedback_path(tree_target: torch.Tensor, path_idx: torch.Tensor, drafter:
                                 ws_bytes if workspace is not None else 0, _ptr(dev_status),
                                 _stream(stream))
     _check(st, "hs_feedback_path")
+    return alpha, e_len
+
+
+def _topl_outputs(drafter, alpha, e_len, workspace):
+    alpha, e_len, _, _ = _feedback_outputs(drafter, alpha, e_len, None, False, with_workspace=False)
+    N, B, P, V = drafter.shape
+    ws_bytes = lib().hs_feedback_topl_workspace_size(N, B, P, V)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 1), device=drafter.device, dtype=torch.uint8)
+    return alpha, e_len, workspace, ws_bytes
+
+
+def hs_feedback_topl(target: torch.Tensor, drafter: torch.Tensor, L: int,
+                     temperature: float = 1.0, greedy: bool = False, alpha=None, e_len=None,
+                     workspace=None, dev_status=None, stream=None):
+    """Draft-tree feedback (Thm 2): alpha [N,B,P] = the target's mass on the
+    drafter's top-L tokens (greedy: whether its argmax is among them), and
+    e_len [N,B] (Thm 3)."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(target, "target", drafter.dtype, (B, P, V))
+    alpha, e_len, workspace, ws_bytes = _topl_outputs(drafter, alpha, e_len, workspace)
+    st = lib().hs_feedback_topl(_ptr(target), _ptr(drafter), _dtype_code(drafter), N, B, P, V,
+                                float(temperature), int(bool(greedy)), int(L), _ptr(alpha),
+                                _ptr(e_len), _ptr(workspace), ws_bytes, _ptr(dev_status),
+                                _stream(stream))
+    _check(st, "hs_feedback_topl")
+    return alpha, e_len
+
+
+def hs_feedback_topl_path(tree_target: torch.Tensor, path_idx: torch.Tensor,
+                          drafter: torch.Tensor, L: int, temperature: float = 1.0,
+                          greedy: bool = False, alpha=None, e_len=None, workspace=None,
+                          dev_status=None, stream=None):
+    """As hs_feedback_topl with target row (b,k) = tree_target[b, path_idx[b,k]]."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(tree_target, "tree_target", drafter.dtype)
+    if tree_target.dim() != 3 or tree_target.shape[0] != B or tree_target.shape[2] != V:
+        raise ValueError(f"tree_target must be [B, M, V] = [{B}, M, {V}]")
+    M = tree_target.shape[1]
+    _need(path_idx, "path_idx", torch.int32, (B, P))
+    alpha, e_len, workspace, ws_bytes = _topl_outputs(drafter, alpha, e_len, workspace)
+    st = lib().hs_feedback_topl_path(_ptr(tree_target), _ptr(path_idx), M, _ptr(drafter),
+                                     _dtype_code(drafter), N, B, P, V, float(temperature),
+                                     int(bool(greedy)), int(L), _ptr(alpha), _ptr(e_len),
+                                     _ptr(workspace), ws_bytes, _ptr(dev_status), _stream(stream))
+    _check(st, "hs_feedback_topl_path")
     return alpha, e_len
 
 

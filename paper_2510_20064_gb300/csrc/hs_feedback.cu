@@ -22,6 +22,7 @@
 #include "hs_fused.h"
 #include "hs_greedy.h"
 #include "hs_stream.h"
+#include "hs_topl.h"
 
 namespace hs {
 
@@ -334,8 +335,58 @@ hs_status feedback_common(const void* target, const int32_t* path, int M, const 
   }
 }
 
+// Draft-tree feedback (Thm 2): validation shared by the chain and path entries.
+hs_status topl_common(const void* target, const int32_t* path, int M, const void* drafter,
+                      int dtype, int N, int B, int P, int V, float temperature, int greedy, int L,
+                      float* alpha, float* e_len, void* ws, size_t ws_bytes, int* dev_status,
+                      void* stream) {
+  if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return HS_ERR_INVALID_ARG;
+  if (!sizes_ok(N, B, P, V)) return HS_ERR_INVALID_ARG;
+  if (L < 1) return HS_ERR_INVALID_ARG;
+  if (L > topl::kMaxL) return HS_ERR_UNSUPPORTED;
+  if (V >= (1 << 30)) return HS_ERR_UNSUPPORTED;  // token indices live in 32-bit keys
+  if (!target || !drafter || !alpha) return HS_ERR_INVALID_ARG;
+  if (!greedy && !(isfinite(temperature) && temperature > 0.f)) return HS_ERR_INVALID_ARG;
+  const int esz = elem_bytes(dtype);
+  if (reinterpret_cast<uintptr_t>(target) % esz || reinterpret_cast<uintptr_t>(drafter) % esz ||
+      reinterpret_cast<uintptr_t>(alpha) % 4 || reinterpret_cast<uintptr_t>(e_len) % 4 ||
+      reinterpret_cast<uintptr_t>(dev_status) % 4)
+    return HS_ERR_MISALIGNED;
+  if (!ws || ws_bytes < topl::workspace_bytes(N, B, P, V)) return HS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(ws) % 256) return HS_ERR_MISALIGNED;
+  const float c = kLog2e / (greedy ? 1.f : temperature);
+  return topl::launch(target, path, M, drafter, dtype, N, B, P, V, L, greedy, c, alpha, e_len, ws,
+                      dev_status, static_cast<cudaStream_t>(stream));
+}
+
 }  // namespace
 }  // namespace hs
+
+extern "C" size_t hs_feedback_topl_workspace_size(int N, int B, int P, int V) {
+  if (!hs::sizes_ok(N, B, P, V)) return 0;
+  return hs::align256(hs::topl::workspace_bytes(N, B, P, V));
+}
+
+extern "C" hs_status hs_feedback_topl(const void* target, const void* drafter, int dtype, int N,
+                                      int B, int P, int V, float temperature, int greedy, int L,
+                                      float* alpha, float* e_len, void* workspace,
+                                      size_t workspace_bytes, int* dev_status, void* stream) {
+  return hs::topl_common(target, nullptr, 0, drafter, dtype, N, B, P, V, temperature, greedy, L,
+                         alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" hs_status hs_feedback_topl_path(const void* tree_target, const int32_t* path_idx,
+                                           int M, const void* drafter, int dtype, int N, int B,
+                                           int P, int V, float temperature, int greedy, int L,
+                                           float* alpha, float* e_len, void* workspace,
+                                           size_t workspace_bytes, int* dev_status,
+                                           void* stream) {
+  if (!path_idx || M < 1) return HS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(path_idx) % 4) return HS_ERR_MISALIGNED;
+  if (double(B) * double(M) * double(V) >= 4.6e18) return HS_ERR_INVALID_ARG;
+  return hs::topl_common(tree_target, path_idx, M, drafter, dtype, N, B, P, V, temperature,
+                         greedy, L, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}
 
 extern "C" size_t hs_feedback_workspace_size(int N, int B, int P, int V, int dtype, int greedy) {
   if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return 0;

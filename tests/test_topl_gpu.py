@@ -1,0 +1,174 @@
+"""hs_feedback_topl / hs_feedback_topl_path (Thm 2, EAGLE tree with branching
+L) against the fp64 oracle, through the C ABI.
+
+alpha is the target's probability mass on the drafter's top-L tokens; the
+candidate set depends only on the stored drafter logits, so the greedy
+results (and the sets behind the stochastic ones) must match exactly.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2510_20064_gb300 as hf
+from paper_2510_20064_gb300 import synth
+from parity_util import RTOL_ALPHA, assert_rel, to_np
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+W = synth.WORKLOADS
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    hf.lib()
+    assert torch.cuda.is_available()
+
+
+def run(d, T, greedy, L):
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    if "path" in d:
+        a, e = hf.hs_feedback_topl_path(d["target"], d["path"], d["drafter"], L, T, greedy,
+                                        dev_status=status)
+    else:
+        a, e = hf.hs_feedback_topl(d["target"], d["drafter"], L, T, greedy, dev_status=status)
+    torch.cuda.synchronize()
+    return to_np(a), to_np(e), int(status.item())
+
+
+def oracle_topl(d, T, greedy, L):
+    path = d.get("path")
+    return oracle.get().feedback_topl(synth.storage_numpy(d["target"]),
+                                      synth.storage_numpy(d["drafter"]), T, greedy, L,
+                                      path=None if path is None else path.cpu().numpy())
+
+
+def compare(d, T, greedy, L):
+    a, e, st = run(d, T, greedy, L)
+    ra, re, rst = oracle_topl(d, T, greedy, L)
+    assert rst == 0 and st == hf.HS_OK, (rst, st)
+    if greedy:
+        assert np.array_equal(a, ra), "greedy alpha must be bit-exact"
+        assert np.array_equal(e, re), "greedy e_len must be bit-exact"
+    else:
+        assert_rel(a, ra, RTOL_ALPHA, f"alpha L={L}")
+        assert_rel(e, re, RTOL_ALPHA, f"e_len L={L}")
+    return a
+
+
+CASES = [
+    # workload, size overrides (the paper's vocabularies: many chunks, ragged tail)
+    ("qwen3_8b_chain", dict(B=2, N=3, P=3)),
+    ("llama3_batch", dict(B=2, N=4, P=3)),
+    ("tree_path", dict(B=2, N=3)),
+    ("tiny_chain", {}),
+]
+
+
+@pytest.mark.parametrize("name,sizes", CASES, ids=[c[0] for c in CASES])
+@pytest.mark.parametrize("L", [1, 3, 10, 16])
+def test_topl_matches_oracle(name, sizes, L):
+    w = W[name]
+    d = synth.make_inputs(w, device=DEV, seed=700 + L, **sizes)
+    for greedy in (False, True):
+        compare(d, w.temperature, greedy, L)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
+def test_topl_dtypes_and_ragged_vocab(dtype):
+    w = synth.Workload("rag", N=2, B=2, P=3, V=20001, dtype=dtype, temperature=0.8,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=11)
+    for L in (2, 16):
+        for greedy in (False, True):
+            compare(d, 0.8, greedy, L)
+
+
+def test_topl_ties_and_masks():
+    """Integer logits (many ties at the L boundary) and -inf masked tokens:
+    the lower index must win, exactly as the oracle ranks."""
+    g = torch.Generator(device=DEV).manual_seed(3)
+    N, B, P, V = 3, 2, 3, 9000
+    tgt = torch.randint(-6, 6, (B, P, V), generator=g, device=DEV).float()
+    drf = torch.randint(-6, 6, (N, B, P, V), generator=g, device=DEV).float()
+    drf[torch.rand(N, B, P, V, generator=g, device=DEV) < 0.2] = float("-inf")
+    for dt in (torch.bfloat16, torch.float32):
+        d = {"target": tgt.to(dt).contiguous(), "drafter": drf.to(dt).contiguous()}
+        for L in (1, 5, 16):
+            compare(d, 1.0, True, L)
+            compare(d, 1.0, False, L)
+
+
+def test_topl_adversarial_order():
+    """Ascending drafter logits make every token displace a kept one (the
+    slow path of the per-thread lists); descending ones reject nearly all."""
+    N, B, P, V = 2, 1, 2, 30000
+    ramp = torch.linspace(-8, 8, V, device=DEV)
+    tgt = torch.randn(B, P, V, generator=torch.Generator(device=DEV).manual_seed(4), device=DEV)
+    drf = torch.stack([ramp, ramp.flip(0)]).reshape(N, 1, 1, V).expand(N, B, P, V)
+    d = {"target": tgt.to(torch.bfloat16).contiguous(),
+         "drafter": drf.to(torch.bfloat16).contiguous()}
+    for L in (1, 7, 16):
+        for greedy in (False, True):
+            compare(d, 1.0, greedy, L)
+
+
+def test_topl_special_cases():
+    w = synth.Workload("small", N=2, B=2, P=4, V=10, dtype="bf16", temperature=1.0,
+                       target="gauss", sigma="tiny")
+    d = synth.make_inputs(w, device=DEV, seed=5)
+    a, e, st = run(d, 1.0, False, 16)          # L >= V: every token is a child
+    assert st == hf.HS_OK and np.all(np.abs(a - 1.0) < 1e-6)
+    a1, _, _ = run(d, 1.0, True, 1)            # L = 1, greedy: hs_feedback's greedy rule
+    ag, _ = hf.hs_feedback(d["target"], d["drafter"], 1.0, True)
+    assert np.array_equal(a1, to_np(ag))
+
+
+def test_topl_nonfinite_and_bad_path():
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, B=2, N=3, P=3, V=5000)
+    d["drafter"][1, 0, 2, 17] = float("nan")
+    d["drafter"][2, 1, 0, :] = float("-inf")
+    d["target"][1, 1, 4999] = float("inf")
+    for greedy in (False, True):
+        a, e, st = run(d, 1.0, greedy, 4)
+        ra, re, rst = oracle_topl(d, 1.0, greedy, 4)
+        assert st == hf.HS_ERR_NONFINITE and rst == oracle.NONFINITE
+        assert np.array_equal(np.isnan(a), np.isnan(ra))
+    t = W["tree_path"]
+    dt = synth.make_inputs(t, device=DEV, B=2, N=2)
+    dt["path"][1, 2] = 999
+    a, e, st = run(dt, 1.0, False, 4)
+    assert st == hf.HS_ERR_INVALID_ARG and np.all(np.isnan(a[:, 1, 2]))
+
+
+def test_topl_argument_errors():
+    d = synth.make_inputs(W["tiny_chain"], device=DEV)
+    for L in (0, 17):
+        with pytest.raises(hf.HedgeFBError):
+            hf.hs_feedback_topl(d["target"], d["drafter"], L, 1.0, False)
+
+
+@pytest.mark.parametrize("name", ["llama3_batch", "tree_path"])
+def test_topl_full_size_sampled(name):
+    """The benchmark's sizes, sampled (i, b, k) against the oracle pair by pair."""
+    w = W[name]
+    d = synth.make_inputs(w, device=DEV, seed=9)
+    L = 10
+    o = oracle.get()
+    path = d.get("path")
+    rng = np.random.default_rng(0)
+    samples = [(int(rng.integers(w.N)), int(rng.integers(w.B)), int(rng.integers(w.P)))
+               for _ in range(6)]
+    for greedy in (False, True):
+        a, e, st = run(d, w.temperature, greedy, L)
+        assert st == hf.HS_OK
+        for (i, b, k) in samples:
+            trow = d["target"][b, int(path[b, k])] if path is not None else d["target"][b, k]
+            ra, _ = o.alpha_topl(synth.storage_numpy(trow),
+                                 synth.storage_numpy(d["drafter"][i, b, k]), w.temperature,
+                                 greedy, L)
+            if greedy:
+                assert a[i, b, k] == ra
+            else:
+                assert abs(a[i, b, k] - ra) <= RTOL_ALPHA * abs(ra), (i, b, k, a[i, b, k], ra)
