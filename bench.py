@@ -7,7 +7,11 @@ the next choice) on one batch of seeded synthetic logits already resident in
 HBM.  Prints ONE JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
-                  [--mode stochastic|greedy] [--impl ours|reference]
+                  [--mode stochastic|greedy|topl] [--branch-l L]
+                  [--impl ours|reference]
+
+--mode topl runs the draft-tree feedback (Thm 2: the drafter proposes its L
+most likely tokens as a node's children) with a stochastic target.
 
 Timing: the K steps run as CUDA-graph replays on one stream, bracketed by
 CUDA events after a barrier + synchronize; inputs rotate over enough buffer
@@ -47,7 +51,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=5000)
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    ap.add_argument("--mode", choices=("stochastic", "greedy"), default="stochastic")
+    ap.add_argument("--mode", choices=("stochastic", "greedy", "topl"), default="stochastic")
+    ap.add_argument("--branch-l", type=int, default=10,
+                    help="children per node of the draft tree (--mode topl)")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
@@ -138,6 +144,7 @@ KERNEL_SOURCES = {
     "stochastic": ("hs_common.cuh", "hs_feedback.cu", "hs_fused.cu", "hs_fused.h",
                    "hs_stream.cu", "hs_stream.h"),
     "greedy": ("hs_common.cuh", "hs_feedback.cu", "hs_greedy.cu", "hs_greedy.h"),
+    "topl": ("hs_common.cuh", "hs_feedback.cu", "hs_topl.cu", "hs_topl.h"),
 }
 
 
@@ -174,12 +181,21 @@ def profiled_traffic(workload: str, mode: str):
 
 # ---- CPU oracle baseline ------------------------------------------------------
 
-def oracle_sample(w, sets, greedy, budget_s=10.0):
+def oracle_alpha(o, w, args):
+    """The oracle's per-pair feedback for the bench's mode."""
+    if args.mode == "topl":
+        return lambda t, d: o.alpha_topl(t, d, w.temperature, False, args.branch_l)
+    greedy = args.mode == "greedy"
+    return lambda t, d: o.alpha_pair(t, d, w.temperature, greedy)
+
+
+def oracle_sample(w, sets, args, budget_s=10.0):
     """The fp64 C oracle (single-threaded, as it stands) on whole (b,k)
     tiles of the first input set until ~budget_s seconds of CPU work."""
     import oracle
     from paper_2510_20064_gb300 import synth
     o = oracle.get()
+    pair = oracle_alpha(o, w, args)
     d = sets[0]
     t_all = synth.storage_numpy(d["target"])
     path = d.get("path")
@@ -192,7 +208,7 @@ def oracle_sample(w, sets, greedy, budget_s=10.0):
         drows = synth.storage_numpy(d["drafter"][:, b, k])
         t0 = time.perf_counter()
         for i in range(w.N):
-            o.alpha_pair(trow, drows[i], w.temperature, greedy)
+            pair(trow, drows[i])
         t_used += time.perf_counter() - t0
         evals += w.N * w.V
         tiles += 1
@@ -221,6 +237,7 @@ def run_ours(args):
 
     w = synth.WORKLOADS[args.workload]
     greedy = args.mode == "greedy"
+    topl = args.mode == "topl"
     learner = hf.HS_HEDGE if w.learner == "hedge" else hf.HS_NORMALHEDGE
     N, B, P, V = w.N, w.B, w.P, w.V
     props = torch.cuda.get_device_properties(dev)
@@ -232,7 +249,8 @@ def run_ours(args):
     stream = torch.cuda.Stream(device=dev)
     alpha = torch.empty(N, B, P, device=dev)
     e_len = torch.empty(N, B, device=dev)
-    ws_bytes = hf.hs_feedback_workspace_size(N, B, P, V, synth.DTYPES[w.dtype], greedy)
+    ws_bytes = (hf.hs_feedback_topl_workspace_size(N, B, P, V) if topl else
+                hf.hs_feedback_workspace_size(N, B, P, V, synth.DTYPES[w.dtype], greedy))
     ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     state = torch.zeros(N, B, device=dev)
@@ -241,7 +259,15 @@ def run_ours(args):
     eta = w.eta if w.eta else math.sqrt(8 * math.log(max(N, 2)) / 2000)
 
     def feedback(d):
-        if "path" in d:
+        if topl and "path" in d:
+            hf.hs_feedback_topl_path(d["target"], d["path"], d["drafter"], args.branch_l,
+                                     w.temperature, False, alpha=alpha, e_len=e_len,
+                                     workspace=ws, dev_status=status, stream=stream)
+        elif topl:
+            hf.hs_feedback_topl(d["target"], d["drafter"], args.branch_l, w.temperature, False,
+                                alpha=alpha, e_len=e_len, workspace=ws, dev_status=status,
+                                stream=stream)
+        elif "path" in d:
             hf.hs_feedback_path(d["target"], d["path"], d["drafter"], w.temperature, greedy,
                                 alpha=alpha, e_len=e_len, workspace=ws, dev_status=status,
                                 stream=stream)
@@ -333,11 +359,12 @@ def run_ours(args):
     peak, peak_src = measured_hbm_peak()
     fb_avg = t_fb / args.steps
     achieved = w.bytes_per_call / fb_avg / 1e9
-    launches_step = hf.hs_feedback_kernel_count(N, B, P, V, synth.DTYPES[w.dtype], greedy) + 1
+    launches_step = 1 + (hf.hs_feedback_topl_kernel_count(N, B, P, V) if topl else
+                         hf.hs_feedback_kernel_count(N, B, P, V, synth.DTYPES[w.dtype], greedy))
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cpu = oracle_sample(w, sets, greedy)
+        cpu = oracle_sample(w, sets, args)
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -348,6 +375,7 @@ def run_ours(args):
                     "(no dataset, no trained weights)",
             "config": {"workload": w.name, "N": N, "B": B, "K": w.K, "V": V,
                        "temperature": None if greedy else w.temperature, "mode": args.mode,
+                       "branch_l": args.branch_l if topl else None,
                        "learner": "hedge" if learner == hf.HS_HEDGE else "normalhedge",
                        "loss": "length", "l2": f"{n_sets} rotating input sets "
                        f"({n_sets * w.bytes_per_call / 2**20:.0f} MiB > 2x L2 {l2 / 2**20:.0f} MiB)",
@@ -378,9 +406,9 @@ def run_reference(args):
     import torch
     from paper_2510_20064_gb300 import synth
     w = synth.WORKLOADS[args.workload]
-    greedy = args.mode == "greedy"
     d = synth.make_inputs(w, device="cpu", B=min(w.B, 2))
     o = oracle.get()
+    pair = oracle_alpha(o, w, args)
     t_all = synth.storage_numpy(d["target"])
     path = d.get("path")
     path_np = None if path is None else path.numpy()
@@ -391,7 +419,7 @@ def run_reference(args):
         trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
         drows = synth.storage_numpy(d["drafter"][:, b, k])
         for i in range(w.N):
-            o.alpha_pair(trow, drows[i], w.temperature, greedy)
+            pair(trow, drows[i])
 
     for s in range(args.warmup):
         one(s)
@@ -409,7 +437,7 @@ def run_reference(args):
         "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "N": w.N, "B": w.B, "K": w.K, "V": w.V,
-                   "mode": args.mode},
+                   "mode": args.mode, "branch_l": args.branch_l if args.mode == "topl" else None},
         "cpu_baseline": {"value": value, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "evals/s", "h2d_bytes_per_step": 0,

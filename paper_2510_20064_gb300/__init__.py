@@ -38,6 +38,7 @@ SIGNATURES = {
     "hs_feedback_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_static": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _P], _I),
     "hs_feedback_topl_workspace_size": ([_I, _I, _I, _I], _Z),
+    "hs_feedback_topl_kernel_count": ([_I, _I, _I, _I], _I),
     "hs_feedback_topl": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_topl_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z,
                                _P, _P], _I),
@@ -121,6 +122,14 @@ def hs_feedback_workspace_size(N: int, B: int, P: int, V: int, dtype, greedy: bo
 def hs_feedback_kernel_count(N: int, B: int, P: int, V: int, dtype, greedy: bool) -> int:
     code = dtype if isinstance(dtype, int) else _DTYPES[dtype]
     return int(lib().hs_feedback_kernel_count(N, B, P, V, code, int(bool(greedy))))
+
+
+def hs_feedback_topl_kernel_count(N: int, B: int, P: int, V: int) -> int:
+    return int(lib().hs_feedback_topl_kernel_count(N, B, P, V))
+
+
+def hs_feedback_topl_workspace_size(N: int, B: int, P: int, V: int) -> int:
+    return int(lib().hs_feedback_topl_workspace_size(N, B, P, V))
 
 
 def _feedback_outputs(drafter, alpha, e_len, workspace, greedy, with_workspace=True):

@@ -367,6 +367,11 @@ extern "C" size_t hs_feedback_topl_workspace_size(int N, int B, int P, int V) {
   return hs::align256(hs::topl::workspace_bytes(N, B, P, V));
 }
 
+extern "C" int hs_feedback_topl_kernel_count(int N, int B, int P, int V) {
+  if (!hs::sizes_ok(N, B, P, V)) return 0;
+  return hs::topl::kernel_count(N, B, P, V);
+}
+
 extern "C" hs_status hs_feedback_topl(const void* target, const void* drafter, int dtype, int N,
                                       int B, int P, int V, float temperature, int greedy, int L,
                                       float* alpha, float* e_len, void* workspace,

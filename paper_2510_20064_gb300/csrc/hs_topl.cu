@@ -192,8 +192,7 @@ struct Vec<HS_BF16> {
     const uint32_t x = (q & 4) ? hi : lo;
     return __uint_as_float((x << (16 - 16 * (q & 1))) & 0xffff0000u);
   }
-  __device__ static __forceinline__ float max(uint4 w) {
-    const uint32_t m = pmax(pmax(w.x, w.y), pmax(w.z, w.w));
+  __device__ static __forceinline__ float wfloat(uint32_t m) {  // max of a packed pair
     return max_nan(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
   }
 };
@@ -219,8 +218,7 @@ struct Vec<HS_FP16> {
     const uint32_t x = (q & 4) ? hi : lo;
     return __half2float(__ushort_as_half(static_cast<unsigned short>(x >> (16 * (q & 1)))));
   }
-  __device__ static __forceinline__ float max(uint4 w) {
-    const uint32_t m = pmax(pmax(w.x, w.y), pmax(w.z, w.w));
+  __device__ static __forceinline__ float wfloat(uint32_t m) {
     return max_nan(half(m, 0), half(m, 1));
   }
 };
@@ -236,10 +234,10 @@ struct Vec<HS_FP32> {
     const uint32_t lo = (q & 1) ? w.y : w.x, hi = (q & 1) ? w.w : w.z;
     return __uint_as_float((q & 2) ? hi : lo);
   }
-  __device__ static __forceinline__ float max(uint4 w) {
-    return max_nan(max_nan(__uint_as_float(w.x), __uint_as_float(w.y)),
-                   max_nan(__uint_as_float(w.z), __uint_as_float(w.w)));
+  __device__ static __forceinline__ uint32_t pmax(uint32_t a, uint32_t b) {
+    return __float_as_uint(max_nan(__uint_as_float(a), __uint_as_float(b)));
   }
+  __device__ static __forceinline__ float wfloat(uint32_t m) { return __uint_as_float(m); }
 };
 
 // Vector of the row starting at logit v (-inf past the end of the row).
@@ -356,15 +354,19 @@ __global__ void __launch_bounds__(kThreads) topl_kernel(
       for (int u = 0; u < kUnroll; ++u)
         nxt[u] = load_vec<DT, VEC>(row, base + kWarpStep + int64_t(u * 32 + l) * kN, lim);
     }
-    float vm[kUnroll];
+    // NaN-propagating maxima: one packed word per vector, then the lane's
+    uint32_t pw[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) vm[u] = Vec<DT>::max(cur[u]);
-    float lm = vm[0];
+    for (int u = 0; u < kUnroll; ++u)
+      pw[u] = Vec<DT>::pmax(Vec<DT>::pmax(cur[u].x, cur[u].y), Vec<DT>::pmax(cur[u].z, cur[u].w));
+    uint32_t lw = pw[0];
 #pragma unroll
-    for (int u = 1; u < kUnroll; ++u) lm = max_nan(lm, vm[u]);
+    for (int u = 1; u < kUnroll; ++u) lw = Vec<DT>::pmax(lw, pw[u]);
+    const float lm = Vec<DT>::wfloat(lw);
     bad |= (lm != lm) || lm == INFINITY;
     any_finite |= lm > -INFINITY;
     uint64_t floor_key = tk;  // candidates must beat this key
+    bool warm = false;
     if (tk == 0ull) {
       // list not full: the L-th largest lane maximum of this step, as a key
       // below every key of that value, bounds the step's top L from below
@@ -378,51 +380,69 @@ __global__ void __launch_bounds__(kThreads) topl_kernel(
         if (l == __ffs(who) - 1) lk = 0u;  // drop one lane holding it
       }
       floor_key = th == 0u ? 0ull : (uint64_t(th) << 32) - 1;
+      warm = true;
     }
-    // vectors that may hold a key above the floor.  The floor's value part
-    // is compared strictly: in the first step the floor sits just below the
-    // bound's value, and later it is a key from an earlier step, whose index
-    // is below every index of this step, so an equal value cannot beat it.
-    uint32_t cmask = 0u;
+    // The floor's value as a float (order keys up to okey(-inf) = 0x007fffff
+    // stand for -inf; the ones below it are NaN patterns).  A key above the
+    // floor has a value >= it; NaN fails every compare.  Below a warm-up
+    // floor a value equal to the bound enters; below a key from an earlier
+    // step an equal value cannot (its index is larger), so there the
+    // vector test is strict.
+    const uint32_t fh0 = uint32_t(floor_key >> 32);
+    const float fz0 = fh0 <= 0x007fffffu ? -INFINITY : ofloat(fh0);
+    if (__any_sync(0xffffffffu, warm ? lm >= fz0 : lm > fz0)) {
+      uint32_t cmask = 0u;  // vectors that may hold a key above the floor
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u)
-      if (vm[u] == vm[u] && okey(vm[u]) > uint32_t(floor_key >> 32)) cmask |= 1u << u;
-    uint64_t ub = ~0ull;  // keys already inserted from this step are >= ub
-    while (__any_sync(0xffffffffu, cmask != 0u)) {
-      // a key above the floor has a value >= the floor's value as a float
-      // (NaN fails the compare); only those logits get the exact key test.
-      // Order keys up to okey(-inf) = 0x007fffff stand for -inf (the ones
-      // below it are NaN patterns).
-      const uint32_t fh = uint32_t(floor_key >> 32);
-      const float fz = fh <= 0x007fffffu ? -INFINITY : ofloat(fh);
-      uint64_t best = 0ull;
-      for (uint32_t m = cmask; m != 0u; m &= m - 1u) {
-        const int u = __ffs(m) - 1;
-        uint4 wv = cur[0];
-#pragma unroll
-        for (int j = 1; j < kUnroll; ++j)
-          if (u == j) wv = cur[j];
-        const int64_t v0 = base + int64_t(u * 32 + l) * kN;
-        uint32_t em = 0u;
-#pragma unroll
-        for (int q = 0; q < kN; ++q) em |= (Vec<DT>::at(wv, q) >= fz ? 1u : 0u) << q;
-        for (; em != 0u; em &= em - 1u) {
-          const int q = __ffs(em) - 1;
-          const float z = Vec<DT>::at_dyn(wv, q);
-          const uint64_t k = token_key(z, v0 + q);
-          if (v0 + q < lim && k > floor_key && k < ub && k > best) best = k;
-        }
+      for (int u = 0; u < kUnroll; ++u) {
+        const float vm = Vec<DT>::wfloat(pw[u]);
+        if (warm ? vm >= fz0 : vm > fz0) cmask |= 1u << u;
       }
-      if (best == 0ull) cmask = 0u;  // nothing of this lane can enter any more
-      const uint64_t K = warp_best(best);
-      if (K == 0ull) break;
-      // insert K: lanes above its slot keep theirs, the rest shift down one
-      const int slot = __popc(__ballot_sync(0xffffffffu, l < L && key > K));
-      const uint64_t above = shfl_up_u64(key);
-      if (l < L) key = l < slot ? key : (l == slot ? K : above);
-      tk = shfl_u64(key, L - 1);
-      if (tk > floor_key) floor_key = tk;
-      ub = K;
+      // Each round, every lane proposes its best key above the floor and
+      // below the last key it had inserted (lub); the proposals enter the
+      // list largest first.  A lane whose proposal is rejected, or that had
+      // no second candidate, is done with this step.
+      uint64_t lub = ~0ull;
+      while (__any_sync(0xffffffffu, cmask != 0u)) {
+        const uint32_t fh = uint32_t(floor_key >> 32);
+        const float fz = fh <= 0x007fffffu ? -INFINITY : ofloat(fh);
+        uint64_t prop = 0ull;
+        int cnt = 0;
+        for (uint32_t m = cmask; m != 0u; m &= m - 1u) {
+          const int u = __ffs(m) - 1;
+          uint4 wv = cur[0];
+#pragma unroll
+          for (int j = 1; j < kUnroll; ++j)
+            if (u == j) wv = cur[j];
+          const int64_t v0 = base + int64_t(u * 32 + l) * kN;
+          uint32_t em = 0u;
+#pragma unroll
+          for (int q = 0; q < kN; ++q) em |= (Vec<DT>::at(wv, q) >= fz ? 1u : 0u) << q;
+          for (; em != 0u; em &= em - 1u) {
+            const int q = __ffs(em) - 1;
+            const uint64_t k = token_key(Vec<DT>::at_dyn(wv, q), v0 + q);
+            if (v0 + q < lim && k > floor_key && k < lub) {
+              ++cnt;
+              if (k > prop) prop = k;
+            }
+          }
+        }
+        if (cnt <= 1) cmask = 0u;  // its only candidate is proposed now (or none)
+        for (;;) {
+          const uint64_t K = warp_best(prop);
+          if (K <= floor_key) break;  // the rest are at or below the floor
+          // insert K: lanes above its slot keep theirs, the rest shift down one
+          const int slot = __popc(__ballot_sync(0xffffffffu, l < L && key > K));
+          const uint64_t above = shfl_up_u64(key);
+          if (l < L) key = l < slot ? key : (l == slot ? K : above);
+          tk = shfl_u64(key, L - 1);
+          if (tk > floor_key) floor_key = tk;
+          if (prop == K) {
+            lub = K;
+            prop = 0ull;
+          }
+        }
+        if (prop != 0ull) cmask = 0u;  // rejected: the lane's other keys are smaller
+      }
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) cur[u] = nxt[u];
@@ -569,6 +589,10 @@ hs_status launch_dt(bool vec, const void* target, const int32_t* path, int M,
 }
 
 }  // namespace
+
+int kernel_count(int N, int B, int P, int V) {
+  return split_of(int64_t(N) * B * P, V) > 1 ? 4 : 3;
+}
 
 size_t workspace_bytes(int N, int B, int P, int V) {
   const int64_t rows = int64_t(N) * B * P;

@@ -17,6 +17,9 @@ constexpr int kMaxL = 16;  // children per node the kernels rank
 // the partial lists of rows split over several warps.
 size_t workspace_bytes(int N, int B, int P, int V);
 
+// Kernels launch() runs with a non-null e_len.
+int kernel_count(int N, int B, int P, int V);
+
 // alpha [N,B,P] (and e_len [N,B] when non-null); c = log2(e) / T.
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
                  int N, int B, int P, int V, int L, int greedy, float c, float* alpha,
