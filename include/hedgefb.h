@@ -151,13 +151,12 @@ hs_status hs_feedback_path(const void* tree_target, const int32_t* path_idx,
 #define HS_MAX_TREE_L 16
 
 /* Bytes of device workspace hs_feedback_topl / hs_feedback_topl_path need
- * (range statistics of the target rows, and partial candidate lists when
- * rows are split over several warps); 0 for invalid sizes. */
+ * (the target rows' share statistics, each drafter row's candidate list and
+ * one counter per (drafter, query)); 0 for invalid sizes. */
 size_t hs_feedback_topl_workspace_size(int N, int B, int P, int V);
 
 /* Number of kernels one hs_feedback_topl / hs_feedback_topl_path call with
- * these sizes and a non-null e_len launches (one fewer with e_len NULL);
- * 0 for invalid sizes. */
+ * these sizes launches (for launch accounting); 0 for invalid sizes. */
 int hs_feedback_topl_kernel_count(int N, int B, int P, int V);
 
 /* Panoramic feedback for an EAGLE draft tree with branching L (Sec. 2.3,

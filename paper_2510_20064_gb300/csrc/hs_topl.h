@@ -13,11 +13,11 @@ namespace topl {
 
 constexpr int kMaxL = 16;  // children per node the kernels rank
 
-// Bytes of workspace launch() needs: one row statistic per target row, and
-// the partial lists of rows split over several warps.
+// Bytes of workspace launch() needs: the target rows' share statistics, the
+// drafter rows' candidate lists, and one counter per (drafter, query).
 size_t workspace_bytes(int N, int B, int P, int V);
 
-// Kernels launch() runs with a non-null e_len.
+// Kernels one launch() runs.
 int kernel_count(int N, int B, int P, int V);
 
 // alpha [N,B,P] (and e_len [N,B] when non-null); c = log2(e) / T.
