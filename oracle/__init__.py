@@ -55,6 +55,12 @@ def _bind(lib):
         "orc_hedge": ([P, I, D, P, P], None),
         "orc_normalhedge": ([P, P, P, I, P, P], I),
         "orc_learner_step": ([P, P, I, I, I, I, I, D, P, P, P, P, P], I),
+        "orc_sample_select": ([P, I, ctypes.c_float], I),
+        "orc_chunk_loss": ([P, I, I], D),
+        "orc_chunk_learner_step": ([P, I, I, I, P, I, I, D, P, P, P, P, P], I),
+        "orc_token_loss": ([P, L, I, I], D),
+        "orc_token_revealed": ([L, I, I, L], L),
+        "orc_token_session": ([P, P, I, I, I, I, I, I, L, I, D, P, P, P, P, P, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -248,6 +254,64 @@ class Oracle:
         if st != OK:
             raise ValueError(f"oracle learner_step rejected its arguments (status {st})")
         return state, weights, loss, sel, pl
+
+
+    # ---- App. B.1 (QFI-D): sampled play; App. B.3 / Sec. 3.2 delayed games ----
+
+    def sample_select(self, w, u: float) -> int:
+        """Inverse-CDF draw from fp32 weights w[N] with uniform u (fp32)."""
+        w = np.ascontiguousarray(w, dtype=np.float32)
+        return int(self.lib.orc_sample_select(_ptr(w), w.shape[0], float(np.float32(u))))
+
+    def chunk_loss(self, gamma, k: int, loss_kind: int) -> float:
+        g = _f64(gamma)
+        return float(self.lib.orc_chunk_loss(_ptr(g), int(k), int(loss_kind)))
+
+    def chunk_learner_step(self, alpha, k_h, loss_kind: int, learner_kind: int, eta: float,
+                           state, weights, selected, played=None):
+        """Chunk-level round with per-query chunk horizon k_h[B]; returns
+        (state, weights, loss, selected, played) as new arrays."""
+        alpha = _f64(alpha)
+        N, B, P = alpha.shape
+        kh = np.ascontiguousarray(k_h, dtype=np.int32)
+        state, weights = _f64(state).copy(), _f64(weights).copy()
+        sel = np.ascontiguousarray(selected, dtype=np.int32).copy()
+        loss = np.empty((N, B), np.float64)
+        pl = None if played is None else _f64(played).copy()
+        st = self.lib.orc_chunk_learner_step(_ptr(alpha), N, B, P, _ptr(kh), int(loss_kind),
+                                             int(learner_kind), float(eta), _ptr(state),
+                                             _ptr(weights), _ptr(loss), _ptr(sel),
+                                             None if pl is None else _ptr(pl))
+        if st != OK:
+            raise ValueError(f"oracle chunk_learner_step rejected its arguments (status {st})")
+        return state, weights, loss, sel, pl
+
+    def token_loss(self, g, s: int, K: int, loss_kind: int) -> float:
+        g = _f64(g)
+        return float(self.lib.orc_token_loss(_ptr(g), int(s), int(K), int(loss_kind)))
+
+    def token_revealed(self, n: int, K: int, loss_kind: int, accept_first: int = 0) -> int:
+        return int(self.lib.orc_token_revealed(int(n), int(K), int(loss_kind), int(accept_first)))
+
+    def token_session(self, alpha, k_h, K: int, loss_kind: int, learner_kind: int, eta: float,
+                      state, weights, sel0, accept_first: int = 0):
+        """Token-level QFI-D session; alpha [H,N,B,P], k_h [H,B].  Returns
+        (state, weights, sel [H,B], played [B], processed [B])."""
+        alpha = _f64(alpha)
+        H, N, B, P = alpha.shape
+        kh = np.ascontiguousarray(k_h, dtype=np.int32)
+        state, weights = _f64(state).copy(), _f64(weights).copy()
+        s0 = np.ascontiguousarray(sel0, dtype=np.int32)
+        sel = np.zeros((H, B), np.int32)
+        played = np.zeros(B, np.float64)
+        done = np.zeros(B, np.int64)
+        st = self.lib.orc_token_session(_ptr(alpha), _ptr(kh), H, N, B, P, int(K), int(loss_kind),
+                                        int(accept_first), int(learner_kind), float(eta),
+                                        _ptr(state), _ptr(weights), _ptr(s0), _ptr(sel),
+                                        _ptr(played), _ptr(done))
+        if st != OK:
+            raise ValueError(f"oracle token_session rejected its arguments (status {st})")
+        return state, weights, sel, played, done
 
 
 _default: Oracle | None = None

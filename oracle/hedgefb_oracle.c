@@ -19,6 +19,11 @@
  *   - App. B.1 remark:       Hedge, w_i <- w_i exp(-eta l_i), normalised
  *   - App. D.6 (Fig. "NormalHedge"): NormalHedge regret update, scale c and
  *                            weights
+ *   - App. B.1 (QFI-D):      a draw "according to p" by the inverse CDF, and
+ *                            the FIFO catch-up of delayed loss vectors
+ *   - App. B.3:              chunk-level losses with the chunk horizon k_h
+ *   - Sec. 3.2 (Fig. "Token-Level Game with Delay"): per-token losses and
+ *                            the rule of when each is revealed
  * Input logits are read as the very bytes the GPU reads: bf16 is widened by
  * a 16-bit shift, fp16 by its IEEE-754 binary16 definition, fp32 as is; all
  * three conversions to double are exact.
@@ -474,5 +479,188 @@ int orc_learner_step(const double* alpha, const double* e_len, int N, int B,
   free(col);
   free(w);
   free(g);
+  return ORC_OK;
+}
+
+/* ---- App. B.1 (QFI-D): playing an action "according to p" -------------- */
+
+/* A draw from the weights by the inverse CDF, with a uniform u in [0, 1)
+ * supplied by the caller: the first i whose running sum w_0 + ... + w_i
+ * exceeds u times the total.  This is an integer decided by floating-point
+ * sums, so it is decided in the kernels' precision: fp32, both sums in index
+ * order, the threshold u * total rounded once.  The running sum can first
+ * exceed the threshold only where it grows, i.e. at a positive weight, so a
+ * zero weight is never drawn; if rounding leaves every running sum at or
+ * below the threshold (u next to 1), the last positive weight is drawn.
+ * Returns -1 for unusable input: u outside [0, 1), a negative, NaN or
+ * infinite weight, or no positive weight. */
+int orc_sample_select(const float* w, int N, float u) {
+  if (!(u >= 0.0f && u < 1.0f)) return -1;
+  float total = 0.0f;
+  for (int i = 0; i < N; ++i) {
+    if (!(w[i] >= 0.0f) || isinf(w[i])) return -1;
+    total += w[i];
+  }
+  if (!(total > 0.0f) || isinf(total)) return -1;
+  const float thr = u * total;
+  float run = 0.0f;
+  int last_pos = -1;
+  for (int i = 0; i < N; ++i) {
+    run += w[i];
+    if (w[i] > 0.0f) last_pos = i;
+    if (run > thr) return i;
+  }
+  return last_pos;
+}
+
+/* ---- App. B.3 chunk-level game with a chunk horizon k_h ----------------- */
+
+/* The losses of one chunk whose chosen drafter had k accepted draft tokens:
+ * Thm 3 with K = k (gamma_1..gamma_k, gamma_{k+1} := 0), and the acceptance
+ * rate over the k tokens.  The positions after k were not verified (the
+ * censoring of Sec. 3.2) and are not read.  k = 0 carries no information:
+ * both losses are 0 (E_len = 1 = K+1, and an empty average is taken as 0). */
+double orc_chunk_loss(const double* gamma, int k, int loss_kind) {
+  if (k <= 0) return 0.0;
+  if (loss_kind == ORC_LOSS_LENGTH) return orc_loss_length(orc_elen_prefix(gamma, k), k);
+  return orc_loss_accept(gamma, k);
+}
+
+/* Base.Update with one loss vector for one query, then Base.Predict (App.
+ * B.1, QFI-D): Hedge keeps the cumulative loss in st and forms w from it;
+ * NormalHedge keeps the regret in st and w = p_t in, p_{t+1} out. */
+static void base_update(int learner_kind, double eta, const double* lv, double* st, double* wt,
+                        int N, int* choice) {
+  if (learner_kind == ORC_HEDGE) {
+    for (int i = 0; i < N; ++i) st[i] = st[i] + lv[i];
+    orc_hedge(st, N, eta, wt, choice);
+  } else {
+    orc_normalhedge(st, lv, wt, N, choice, NULL);
+  }
+}
+
+/* One chunk-level round for B queries (arrays [N,B], alpha [N,B,P]) when
+ * query b's chosen drafter had k_h[b] accepted draft tokens, 0 <= k_h[b] <=
+ * P-1; otherwise as orc_learner_step (loss_out, selected and played alike). */
+int orc_chunk_learner_step(const double* alpha, int N, int B, int P, const int* k_h,
+                           int loss_kind, int learner_kind, double eta, double* state,
+                           double* weights, double* loss_out, int* selected, double* played) {
+  if (N < 1 || B < 1 || P < 1) return ORC_BADARG;
+  for (int b = 0; b < B; ++b)
+    if (k_h[b] < 0 || k_h[b] > P - 1) return ORC_BADARG;
+  double* lv = (double*)malloc(sizeof(double) * (size_t)N);
+  double* st = (double*)malloc(sizeof(double) * (size_t)N);
+  double* wt = (double*)malloc(sizeof(double) * (size_t)N);
+  double* gm = (double*)malloc(sizeof(double) * (size_t)P);
+  for (int b = 0; b < B; ++b) {
+    for (int i = 0; i < N; ++i) {
+      for (int k = 0; k < P; ++k) gm[k] = alpha[((size_t)i * B + b) * P + k];
+      lv[i] = orc_chunk_loss(gm, k_h[b], loss_kind);
+      if (loss_out) loss_out[i * B + b] = lv[i];
+      st[i] = state[i * B + b];
+      wt[i] = weights[i * B + b];
+    }
+    if (played) played[b] = played[b] + lv[selected[b]];
+    int choice = 0;
+    base_update(learner_kind, eta, lv, st, wt, N, &choice);
+    for (int i = 0; i < N; ++i) {
+      state[i * B + b] = st[i];
+      weights[i * B + b] = wt[i];
+    }
+    selected[b] = choice;
+  }
+  free(lv);
+  free(st);
+  free(wt);
+  free(gm);
+  return ORC_OK;
+}
+
+/* ---- Sec. 3.2 token-level game with delay, through QFI-D (App. B.1) ----- */
+
+/* The loss of choosing drafter i at token s (0-based) of a query's token
+ * stream g_i[0..]: the acceptance-rate loss 1 - g_i[s], or the length loss
+ * of a K-token draft starting at s, 1 - E/(K+1) with E from g_i[s..s+K-1]
+ * (Thm 3). */
+double orc_token_loss(const double* g, int64_t s, int K, int loss_kind) {
+  if (loss_kind == ORC_LOSS_ACCEPT) return 1.0 - g[s];
+  return orc_loss_length(orc_elen_prefix(g + s, K), K);
+}
+
+/* How many of a stream's first n tokens have a revealed loss (Fig. "Token-
+ * Level Game with Delay"): at the end of a chunk that ends at token n (1-
+ * based), f_{<=n} is revealed for the acceptance-rate loss and f_{<=n-K} for
+ * the length loss.  With hybrid losses (App. B.5) the first `accept_first`
+ * tokens use the acceptance-rate loss, the rest loss_kind. */
+int64_t orc_token_revealed(int64_t n, int K, int loss_kind, int64_t accept_first) {
+  int64_t late = (loss_kind == ORC_LOSS_LENGTH) ? n - K : n;
+  if (late < 0) late = 0;
+  int64_t early = n < accept_first ? n : accept_first;
+  return late > early ? late : early;
+}
+
+/* A whole token-level session for B queries through QFI-D.  For chunk h =
+ * 0..H-1 and every query b:
+ *   1. catch up: pop every revealed, unprocessed token loss in token order
+ *      (FIFO) and feed it to Base (Update, then Predict);
+ *   2. play: sel[h*B+b] = Base's choice (the last Update's Predict; with no
+ *      Update yet, the caller's initial choice sel0[b]);
+ *   3. the chunk's k_h[h*B+b]+1 verified tokens join the stream, with
+ *      gamma = alpha[h] at positions 0..k_h of (i, b), each recorded as
+ *      played by sel[h*B+b].
+ * alpha [H,N,B,P] (gamma of drafter i at position k of chunk h, b),
+ * k_h [H,B] in 0..P-1; state/weights [N,B] as in orc_learner_step (initial
+ * values in, final out); played [B] (or NULL) += f_s[drafter that played s]
+ * for every processed token s; processed [B] (or NULL) = tokens processed. */
+int orc_token_session(const double* alpha, const int* k_h, int H, int N, int B, int P, int K,
+                      int loss_kind, int64_t accept_first, int learner_kind, double eta,
+                      double* state, double* weights, const int* sel0, int* sel, double* played,
+                      int64_t* processed) {
+  if (N < 1 || B < 1 || P < 1 || H < 0 || K < 1) return ORC_BADARG;
+  for (int64_t x = 0; x < (int64_t)H * B; ++x)
+    if (k_h[x] < 0 || k_h[x] > P - 1) return ORC_BADARG;
+  const int64_t cap = (int64_t)H * P + 1;
+  double* stream = (double*)malloc(sizeof(double) * (size_t)(N * cap));
+  int* who = (int*)malloc(sizeof(int) * (size_t)cap);
+  double* lv = (double*)malloc(sizeof(double) * (size_t)N);
+  double* st = (double*)malloc(sizeof(double) * (size_t)N);
+  double* wt = (double*)malloc(sizeof(double) * (size_t)N);
+  for (int b = 0; b < B; ++b) {
+    int64_t n = 0, done = 0;
+    int choice = sel0[b];
+    for (int i = 0; i < N; ++i) {
+      st[i] = state[i * B + b];
+      wt[i] = weights[i * B + b];
+    }
+    double own = 0.0;
+    for (int h = 0; h < H; ++h) {
+      const int64_t ready = orc_token_revealed(n, K, loss_kind, accept_first);
+      for (; done < ready; ++done) {
+        const int kind = done < accept_first ? ORC_LOSS_ACCEPT : loss_kind;
+        for (int i = 0; i < N; ++i) lv[i] = orc_token_loss(stream + (size_t)i * cap, done, K, kind);
+        own += lv[who[done]];
+        base_update(learner_kind, eta, lv, st, wt, N, &choice);
+      }
+      sel[(size_t)h * B + b] = choice;
+      const int kk = k_h[(size_t)h * B + b];
+      for (int k = 0; k <= kk; ++k) {
+        for (int i = 0; i < N; ++i)
+          stream[(size_t)i * cap + n] = alpha[(((size_t)h * N + i) * B + b) * P + k];
+        who[n] = choice;
+        ++n;
+      }
+    }
+    for (int i = 0; i < N; ++i) {
+      state[i * B + b] = st[i];
+      weights[i * B + b] = wt[i];
+    }
+    if (played) played[b] += own;
+    if (processed) processed[b] = done;
+  }
+  free(stream);
+  free(who);
+  free(lv);
+  free(st);
+  free(wt);
   return ORC_OK;
 }

@@ -608,4 +608,223 @@ def check_feedback_topl_layout(o):
                 assert abs(e[i, b] - want_e) < 1e-12
 
 
+# ---- App. B.1 (QFI-D): sampled play --------------------------------------------
+
+def check_sample_select_searchsorted(o):
+    """The draw is numpy's searchsorted (side='right') of u * total into the
+    fp32 running sums (np.cumsum accumulates in index order), so the first
+    running sum above the threshold; the last positive weight when none is."""
+    rng = np.random.default_rng(60)
+    for _ in range(400):
+        N = int(rng.integers(1, 33))
+        w = rng.random(N).astype(np.float32)
+        w[rng.random(N) < 0.3] = 0.0
+        if not w.any():
+            w[int(rng.integers(N))] = np.float32(0.5)
+        csum = np.cumsum(w, dtype=np.float32)
+        for u in list(rng.random(6).astype(np.float32)) + [np.float32(0.0)]:
+            thr = np.float32(u) * csum[-1]
+            want = int(np.searchsorted(csum, thr, side="right"))
+            if want == N:
+                want = int(np.flatnonzero(w > 0)[-1])
+            got = o.sample_select(w, float(u))
+            assert got == want, (w, u, got, want)
+            assert w[got] > 0
+
+
+def check_sample_select_frequencies(o):
+    """Over many uniforms each drafter is drawn with frequency w_i / sum w
+    (within 5 sigma), including exact zeros for zero weights."""
+    w = np.array([0.05, 0.0, 0.4, 0.15, 0.3, 0.1], np.float32)
+    rng = np.random.default_rng(61)
+    n = 100_000
+    counts = np.zeros(len(w), np.int64)
+    for u in rng.random(n).astype(np.float32):
+        counts[o.sample_select(w, float(u))] += 1
+    p = w / w.sum()
+    sd = np.sqrt(n * p * (1 - p))
+    assert counts[1] == 0
+    assert np.all(np.abs(counts - n * p) <= 5 * sd + 1e-9), counts
+
+
+def check_sample_select_invalid(o):
+    w = np.array([0.3, 0.7], np.float32)
+    for u in (1.0, -0.25, float("nan")):
+        assert o.sample_select(w, u) == -1
+    for bad in ([0.0, 0.0], [0.5, -0.1], [np.inf, 1.0], [np.nan, 1.0]):
+        assert o.sample_select(np.array(bad, np.float32), 0.5) == -1
+    assert o.sample_select(np.array([0.0, 0.0, 1.0], np.float32), 0.0) == 2
+    u_top = float(np.nextafter(np.float32(1.0), np.float32(0.0)))
+    assert o.sample_select(np.array([0.0, 1.0, 0.0], np.float32), u_top) == 1
+
+
+# ---- App. B.3: chunk-level game with a chunk horizon -------------------------------
+
+def check_chunk_loss_reduces_to_fixed_K(o):
+    """k = K is the fixed-horizon loss; k = 1 is 1 - (1 + g1)/2 and 1 - g1;
+    constant gamma a gives E = (1 - a^{k+1})/(1 - a); positions after k are
+    never read; k = 0 gives 0."""
+    rng = np.random.default_rng(62)
+    for _ in range(50):
+        P = int(rng.integers(2, 12))
+        g = rng.random(P)
+        K = P - 1
+        assert o.chunk_loss(g, K, orc.LOSS_LENGTH) == o.loss_length(o.elen_prefix(g[:K]), K)
+        assert o.chunk_loss(g, K, orc.LOSS_ACCEPT) == o.loss_accept(g[:K])
+        assert abs(o.chunk_loss(g, 1, orc.LOSS_LENGTH) - (1 - (1 + g[0]) / 2)) < 1e-15
+        assert abs(o.chunk_loss(g, 1, orc.LOSS_ACCEPT) - (1 - g[0])) < 1e-15
+        k = int(rng.integers(1, P))
+        h = g.copy()
+        h[k:] = rng.random(P - k)
+        for kind in (orc.LOSS_LENGTH, orc.LOSS_ACCEPT):
+            assert o.chunk_loss(g, k, kind) == o.chunk_loss(h, k, kind)
+            assert o.chunk_loss(g, 0, kind) == 0.0
+        a = float(rng.random())
+        e = (1 - a ** (k + 1)) / (1 - a)
+        assert abs(o.chunk_loss(np.full(P, a), k, orc.LOSS_LENGTH) - (1 - e / (k + 1))) < 1e-13
+
+
+def check_chunk_learner_step_matches_fixed_horizon(o):
+    """Query b of a chunk-level round with horizon k_h[b] is the fixed-horizon
+    round on that query's first k_h[b]+1 positions."""
+    rng = np.random.default_rng(63)
+    N, B, P = 5, 6, 7
+    for learner in (orc.HEDGE, orc.NORMALHEDGE):
+        for kind in (orc.LOSS_LENGTH, orc.LOSS_ACCEPT):
+            alpha = rng.random((N, B, P))
+            k_h = rng.integers(1, P, B)
+            state = rng.random((N, B)) * (0.5 if learner == orc.HEDGE else 0.2)
+            weights = rng.dirichlet(np.ones(N), B).T.copy()
+            sel = rng.integers(0, N, B).astype(np.int32)
+            played = rng.random(B)
+            st, w, loss, s2, pl = o.chunk_learner_step(alpha, k_h, kind, learner, 0.3, state,
+                                                        weights, sel, played)
+            for b in range(B):
+                k = int(k_h[b])
+                a_b = alpha[:, b:b + 1, :k + 1]
+                e_b = np.array([[o.elen_prefix(a_b[i, 0, :k])] for i in range(N)])
+                st1, w1, l1, s1, p1 = o.learner_step(a_b, e_b, kind, learner, 0.3,
+                                                     state[:, b:b + 1], weights[:, b:b + 1],
+                                                     sel[b:b + 1], played[b:b + 1])
+                assert np.array_equal(st[:, b], st1[:, 0]) and np.array_equal(w[:, b], w1[:, 0])
+                assert np.array_equal(loss[:, b], l1[:, 0]) and s2[b] == s1[0]
+                assert pl[b] == p1[0]
+
+
+# ---- Sec. 3.2 token-level game with delay, QFI-D (App. B.1) ---------------------------
+
+def check_token_loss_window(o):
+    """The length loss of token s is the chunk loss of a K-token chunk that
+    starts at s; the acceptance loss is 1 - g[s]."""
+    rng = np.random.default_rng(64)
+    g = rng.random(40)
+    for K in (1, 3, 8):
+        for s in range(0, 40 - K):
+            assert o.token_loss(g, s, K, orc.LOSS_LENGTH) == o.chunk_loss(g[s:s + K], K,
+                                                                         orc.LOSS_LENGTH)
+            assert abs(o.token_loss(g, s, K, orc.LOSS_ACCEPT) - (1 - g[s])) < 1e-15
+
+
+def check_token_revealed_paper_rule(o):
+    """Fig. "Token-Level Game with Delay": at the end of a chunk ending at
+    token t the player knows f_{<=t} (acceptance) or f_{<=t-K} (length);
+    hybrid losses reveal the first accept_first tokens early."""
+    assert o.token_revealed(10, 4, orc.LOSS_LENGTH) == 6
+    assert o.token_revealed(3, 4, orc.LOSS_LENGTH) == 0
+    assert o.token_revealed(10, 4, orc.LOSS_ACCEPT) == 10
+    assert o.token_revealed(5, 8, orc.LOSS_LENGTH, accept_first=3) == 3
+    assert o.token_revealed(2, 8, orc.LOSS_LENGTH, accept_first=3) == 2
+    assert o.token_revealed(20, 8, orc.LOSS_LENGTH, accept_first=3) == 12
+
+
+def _session_inputs(rng, H, N, B, P):
+    alpha = rng.random((H, N, B, P))
+    k_h = rng.integers(0, P, (H, B))
+    return alpha, k_h
+
+
+def _stream(alpha, k_h, b):
+    H, N, _, P = alpha.shape
+    return np.concatenate([alpha[h, :, b, :k_h[h, b] + 1] for h in range(H)], axis=1)
+
+
+def check_token_session_hedge_sum(o):
+    """Hedge through QFI-D: the final cumulative loss is the initial one plus
+    the plain sum of the revealed token losses (order does not matter), the
+    weights are Hedge's closed form of it, and the processed count is the
+    revealed count of the stream before the last chunk's tokens."""
+    rng = np.random.default_rng(65)
+    H, N, B, P, K = 9, 4, 3, 5, 4
+    alpha, k_h = _session_inputs(rng, H, N, B, P)
+    for kind, first in ((orc.LOSS_ACCEPT, 0), (orc.LOSS_LENGTH, 0), (orc.LOSS_LENGTH, 5)):
+        state0 = rng.random((N, B))
+        st, w, sel, played, done = o.token_session(alpha, k_h, K, kind, orc.HEDGE, 0.4, state0,
+                                                   np.full((N, B), 1.0 / N), np.zeros(B),
+                                                   accept_first=first)
+        for b in range(B):
+            g = _stream(alpha, k_h, b)
+            n_before_last = g.shape[1] - (k_h[H - 1, b] + 1)
+            ready = o.token_revealed(n_before_last, K, kind, first)
+            assert done[b] == ready
+            tot = np.zeros(N)
+            for s_ in range(ready):
+                if s_ < first or kind == orc.LOSS_ACCEPT:
+                    tot += 1.0 - g[:, s_]
+                else:
+                    csum = np.cumprod(g[:, s_:s_ + K], axis=1).sum(axis=1)
+                    tot += 1.0 - (1.0 + csum) / (K + 1)
+            assert np.allclose(st[:, b], state0[:, b] + tot, rtol=0, atol=1e-12)
+            ww, ss = o.hedge(st[:, b], 0.4)
+            assert np.array_equal(w[:, b], ww) and sel[H - 1, b] == (ss if ready else 0)
+
+
+def check_token_session_normalhedge_fifo(o):
+    """NormalHedge through QFI-D: the revealed losses are fed in token order
+    (FIFO), one NormalHedge round each, before every chunk's choice."""
+    rng = np.random.default_rng(66)
+    H, N, B, P, K = 8, 5, 2, 4, 3
+    alpha, k_h = _session_inputs(rng, H, N, B, P)
+    for kind in (orc.LOSS_ACCEPT, orc.LOSS_LENGTH):
+        st, w, sel, played, done = o.token_session(alpha, k_h, K, kind, orc.NORMALHEDGE, 0.0,
+                                                   np.zeros((N, B)), np.full((N, B), 1.0 / N),
+                                                   np.zeros(B))
+        for b in range(B):
+            g = _stream(alpha, k_h, b)
+            R, p, choice, n, d, own = np.zeros(N), np.full(N, 1.0 / N), 0, 0, 0, 0.0
+            who = []
+            for h in range(H):
+                ready = o.token_revealed(n, K, kind)
+                while d < ready:
+                    f = np.array([o.token_loss(g[i], d, K, kind) for i in range(N)])
+                    own += f[who[d]]
+                    R, p, choice, _ = o.normalhedge(R, f, p)
+                    d += 1
+                assert sel[h, b] == choice
+                who += [choice] * (k_h[h, b] + 1)
+                n += k_h[h, b] + 1
+            assert np.array_equal(st[:, b], R) and np.array_equal(w[:, b], p)
+            assert done[b] == d and abs(played[b] - own) < 1e-12
+
+
+def check_token_session_unrevealed_is_unseen(o):
+    """The choice for chunk h depends only on revealed losses: changing the
+    gamma of tokens whose loss is not yet revealed leaves sel[h] alone."""
+    rng = np.random.default_rng(67)
+    H, N, B, P, K = 6, 4, 1, 5, 4
+    alpha, k_h = _session_inputs(rng, H, N, B, P)
+    k_h[:] = P - 1
+    args = (K, orc.LOSS_LENGTH, orc.HEDGE, 0.5, np.zeros((N, B)), np.full((N, B), 0.25),
+            np.zeros(B))
+    _, _, sel, _, _ = o.token_session(alpha, k_h, *args)
+    # at chunk 3 the stream holds 3*P tokens, of which the first 3*P-K are
+    # revealed; perturb the later ones (they sit in chunk 2)
+    alt = alpha.copy()
+    n3 = 3 * P
+    for t in range(n3 - K + 1, n3):
+        h, k = divmod(t, P)
+        alt[h, :, 0, k] = rng.random(N)
+    _, _, sel2, _, _ = o.token_session(alt, k_h, *args)
+    assert sel2[3, 0] == sel[3, 0]
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

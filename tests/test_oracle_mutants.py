@@ -66,6 +66,21 @@ MUTANTS = {
                                 "e_len[i * B + b] = orc_elen_prefix(gam, P);"),
     "hedge_state_not_cumulative": ("for (int i = 0; i < N; ++i) col[i] += f[i];",
                                    "for (int i = 0; i < N; ++i) col[i] = f[i];"),
+    "sample_at_or_above": ("if (run > thr) return i;", "if (run >= thr) return i;"),
+    "sample_threshold_unscaled": ("const float thr = u * total;", "const float thr = u;"),
+    "chunk_loss_reads_past_horizon": ("return orc_loss_length(orc_elen_prefix(gamma, k), k);",
+                                      "return orc_loss_length(orc_elen_prefix(gamma, k + 1), k);"),
+    "chunk_played_wrong_drafter": ("played[b] = played[b] + lv[selected[b]];",
+                                   "played[b] = played[b] + lv[0];"),
+    "token_window_shifted": ("return orc_loss_length(orc_elen_prefix(g + s, K), K);",
+                             "return orc_loss_length(orc_elen_prefix(g + s + 1, K), K);"),
+    "token_revealed_one_early": ("int64_t late = (loss_kind == ORC_LOSS_LENGTH) ? n - K : n;",
+                                 "int64_t late = (loss_kind == ORC_LOSS_LENGTH) ? n - K + 1 : n;"),
+    "token_hybrid_ignored": ("const int kind = done < accept_first ? ORC_LOSS_ACCEPT : loss_kind;",
+                             "const int kind = loss_kind;"),
+    "token_played_by_drafter_0": ("who[n] = choice;", "who[n] = 0;"),
+    "qfid_hedge_not_cumulative": ("for (int i = 0; i < N; ++i) st[i] = st[i] + lv[i];",
+                                  "for (int i = 0; i < N; ++i) st[i] = lv[i];"),
 }
 
 
