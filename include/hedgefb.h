@@ -239,6 +239,81 @@ hs_status hs_learner_step(const float* alpha, const float* e_len, int N, int B,
                           float* state, float* weights, float* loss_out,
                           int32_t* selected, float* played_loss, void* stream);
 
+/* Sampled play (App. B.1, QFI-D: "play a_t according to p", here by
+ * sampling from p): for query b, the first drafter i whose running sum
+ * weights[0,b] + ... + weights[i,b] exceeds uniforms[b] times the column's
+ * total, both sums in fp32 in index order and the threshold rounded once; a
+ * zero weight is never drawn, and if rounding leaves no running sum above the
+ * threshold the last positive weight is drawn.
+ *   weights   device, [N,B] fp32: finite, >= 0, some positive per column
+ *             (e.g. the weights a learner call wrote).
+ *   uniforms  device, [B] fp32 in [0, 1), from the caller's generator.
+ *   selected  device, out, [B] int32; -1 for a column or uniform outside
+ *             those rules, which also sets *dev_status = HS_ERR_NONFINITE.
+ * Limits: 1 <= N <= HS_MAX_LEARNER_N, B >= 1. */
+hs_status hs_sample_select(const float* weights, int N, int B, const float* uniforms,
+                           int32_t* selected, int* dev_status, void* stream);
+
+/* Chunk-level learner round with a chunk horizon (App. B.3, game "Chunk-
+ * Level Game"; Sec. 3.2 on censoring): as hs_learner_step, but query b's
+ * chosen drafter had k_h[b] accepted draft tokens, so only positions
+ * 1..k_h[b] were verified and the losses use those alone (Thm 3 with
+ * K = k_h[b]):
+ *   HS_LOSS_LENGTH  f = 1 - (1 + sum_{k<=k_h} prod_{j<=k} alpha_j)/(k_h+1)
+ *   HS_LOSS_ACCEPT  f = (1/k_h) sum_{k<=k_h} (1 - alpha_k)
+ * and k_h[b] = 0 gives f = 0 (no information).  e_len is not an input: it is
+ * formed from alpha.
+ *   k_h       device, [B] int32, 0 <= k_h[b] <= P-1; a query outside that
+ *             range keeps its state and sets *dev_status =
+ *             HS_ERR_INVALID_ARG.
+ * Other arguments as hs_learner_step (loss_out and played_loss may be NULL).
+ */
+hs_status hs_chunk_learner_step(const float* alpha, const int32_t* k_h, int N, int B,
+                                int P, int loss_kind, int learner, float eta,
+                                float* state, float* weights, float* loss_out,
+                                int32_t* selected, float* played_loss, int* dev_status,
+                                void* stream);
+
+/* Token-level game with delay (Sec. 3.2, Fig. "Token-Level Game with Delay")
+ * run through QFI-D (App. B.1).  Each query keeps a stream of its verified
+ * tokens' acceptance probabilities in a caller-owned ring:
+ *   gamma_ring  device, [B,H,N] fp32: gamma of drafter i at token s (0-based)
+ *               of query b sits at [b, s mod H, i];
+ *   who_ring    device, [B,H] int32: the drafter that played token s;
+ *   n_tok       device, [B] int64: tokens in the stream (start at 0);
+ *   n_done      device, [B] int64: tokens whose loss the learner consumed
+ *               (start at 0).
+ * hs_token_append, after a chunk's feedback: the chunk's k_h[b] accepted
+ * draft tokens and the target's token that ends it join the stream with
+ * gamma_i = alpha[i,b,0..k_h[b]], played by selected[b].  k_h as in
+ * hs_chunk_learner_step.  A query whose ring would overwrite unconsumed
+ * tokens (n_tok + k_h + 1 - n_done > H) is not appended and sets *dev_status
+ * = HS_ERR_UNSUPPORTED.  Size the ring H >= K + 2P to never meet this with
+ * one learner call per chunk. */
+hs_status hs_token_append(const float* alpha, const int32_t* k_h, int N, int B, int P,
+                          const int32_t* selected, float* gamma_ring, int32_t* who_ring,
+                          int H, int64_t* n_tok, const int64_t* n_done, int* dev_status,
+                          void* stream);
+
+/* hs_token_learner_step, before a chunk's choice: QFI-D's catch-up.  Every
+ * token loss that is revealed and not yet consumed is fed to the base
+ * learner (HS_HEDGE or HS_NORMALHEDGE, state and weights as in
+ * hs_learner_step) in token order, one round each; selected[b] becomes the
+ * last round's choice (unchanged when nothing was revealed).  Token s's loss
+ * is 1 - gamma_s (HS_LOSS_ACCEPT), or 1 - E/(K+1) with E = 1 +
+ * sum_{k=1..K} prod_{j<k} gamma_{s+j} (HS_LOSS_LENGTH, Thm 3 for a K-token
+ * draft starting at s).  With n tokens in the stream, f_s is revealed for
+ * s < n (acceptance) or s < n - K (length), as in the figure; hybrid losses
+ * (App. B.5): tokens s < accept_first use the acceptance loss and are
+ * revealed at once.  played_loss (or NULL) [B] += f_s[the drafter that
+ * played s] for each consumed token.  1 <= K <= H. */
+hs_status hs_token_learner_step(const float* gamma_ring, const int32_t* who_ring, int N,
+                                int B, int H, const int64_t* n_tok, int64_t* n_done,
+                                int K, int loss_kind, int64_t accept_first, int learner,
+                                float eta, float* state, float* weights,
+                                int32_t* selected, float* played_loss, int* dev_status,
+                                void* stream);
+
 #ifdef __cplusplus
 }
 #endif

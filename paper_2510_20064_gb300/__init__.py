@@ -29,6 +29,7 @@ _DTYPES = {torch.bfloat16: HS_BF16, torch.float16: HS_FP16, torch.float32: HS_FP
 
 # argument/return types of every exported symbol (mirrors include/hedgefb.h)
 _P, _I, _F, _Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+_L = ctypes.c_int64
 SIGNATURES = {
     "hs_status_string": ([_I], ctypes.c_char_p),
     "hs_version": ([], _I),
@@ -45,6 +46,11 @@ SIGNATURES = {
     "hs_hedge_update": ([_P, _I, _I, _F, _P, _P, _P], _I),
     "hs_normalhedge_update": ([_P, _P, _P, _I, _I, _P, _P], _I),
     "hs_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P], _I),
+    "hs_sample_select": ([_P, _I, _I, _P, _P, _P, _P], _I),
+    "hs_chunk_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P], _I),
+    "hs_token_append": ([_P, _P, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P], _I),
+    "hs_token_learner_step": ([_P, _P, _I, _I, _I, _P, _P, _I, _I, _L, _I, _F, _P, _P, _P, _P,
+                               _P, _P], _I),
 }
 
 
@@ -298,4 +304,89 @@ def hs_learner_step(alpha: torch.Tensor, e_len: torch.Tensor, loss_kind: int, le
                                  float(eta), _ptr(state), _ptr(weights), _ptr(loss_out),
                                  _ptr(selected), _ptr(played_loss), _stream(stream)),
            "hs_learner_step")
+    return state, weights, selected
+
+
+# ---- delayed feedback and sampled play (App. B.1, B.3, B.5; Sec. 3.2) -------------
+
+def hs_sample_select(weights: torch.Tensor, uniforms: torch.Tensor, selected=None,
+                     dev_status=None, stream=None) -> torch.Tensor:
+    """Inverse-CDF draw per query from weights [N,B] with uniforms [B]."""
+    _need(weights, "weights", torch.float32)
+    N, B = weights.shape
+    _need(uniforms, "uniforms", torch.float32, (B,))
+    if selected is None:
+        selected = torch.empty(B, dtype=torch.int32, device=weights.device)
+    _need(selected, "selected", torch.int32, (B,))
+    _check(lib().hs_sample_select(_ptr(weights), N, B, _ptr(uniforms), _ptr(selected),
+                                  _ptr(dev_status), _stream(stream)), "hs_sample_select")
+    return selected
+
+
+def hs_chunk_learner_step(alpha: torch.Tensor, k_h: torch.Tensor, loss_kind: int, learner: int,
+                          eta: float, state: torch.Tensor, weights: torch.Tensor,
+                          selected: torch.Tensor, loss_out=None, played_loss=None,
+                          dev_status=None, stream=None):
+    """Chunk-level round with per-query chunk horizon k_h [B] int32, in place."""
+    _need(alpha, "alpha", torch.float32)
+    N, B, P = alpha.shape
+    _need(k_h, "k_h", torch.int32, (B,))
+    _need(state, "state", torch.float32, (N, B))
+    _need(weights, "weights", torch.float32, (N, B))
+    _need(selected, "selected", torch.int32, (B,))
+    if loss_out is not None:
+        _need(loss_out, "loss_out", torch.float32, (N, B))
+    if played_loss is not None:
+        _need(played_loss, "played_loss", torch.float32, (B,))
+    _check(lib().hs_chunk_learner_step(_ptr(alpha), _ptr(k_h), N, B, P, int(loss_kind),
+                                       int(learner), float(eta), _ptr(state), _ptr(weights),
+                                       _ptr(loss_out), _ptr(selected), _ptr(played_loss),
+                                       _ptr(dev_status), _stream(stream)),
+           "hs_chunk_learner_step")
+    return state, weights, selected
+
+
+class TokenStream:
+    """Device state of the token-level game with delay for B queries: the
+    gamma ring [B,H,N], the ring of playing drafters [B,H] and the token
+    counters; hs_token_append / hs_token_learner_step work on it in place."""
+
+    def __init__(self, N: int, B: int, H: int, device):
+        self.N, self.B, self.H = N, B, H
+        self.gamma = torch.zeros(B, H, N, dtype=torch.float32, device=device)
+        self.who = torch.zeros(B, H, dtype=torch.int32, device=device)
+        self.n_tok = torch.zeros(B, dtype=torch.int64, device=device)
+        self.n_done = torch.zeros(B, dtype=torch.int64, device=device)
+
+
+def hs_token_append(ts: TokenStream, alpha: torch.Tensor, k_h: torch.Tensor,
+                    selected: torch.Tensor, dev_status=None, stream=None) -> None:
+    _need(alpha, "alpha", torch.float32)
+    N, B, P = alpha.shape
+    assert (N, B) == (ts.N, ts.B)
+    _need(k_h, "k_h", torch.int32, (B,))
+    _need(selected, "selected", torch.int32, (B,))
+    _check(lib().hs_token_append(_ptr(alpha), _ptr(k_h), N, B, P, _ptr(selected),
+                                 _ptr(ts.gamma), _ptr(ts.who), ts.H, _ptr(ts.n_tok),
+                                 _ptr(ts.n_done), _ptr(dev_status), _stream(stream)),
+           "hs_token_append")
+
+
+def hs_token_learner_step(ts: TokenStream, K: int, loss_kind: int, learner: int, eta: float,
+                          state: torch.Tensor, weights: torch.Tensor, selected: torch.Tensor,
+                          accept_first: int = 0, played_loss=None, dev_status=None,
+                          stream=None):
+    """QFI-D catch-up on the revealed token losses, in place."""
+    N, B = ts.N, ts.B
+    _need(state, "state", torch.float32, (N, B))
+    _need(weights, "weights", torch.float32, (N, B))
+    _need(selected, "selected", torch.int32, (B,))
+    if played_loss is not None:
+        _need(played_loss, "played_loss", torch.float32, (B,))
+    _check(lib().hs_token_learner_step(_ptr(ts.gamma), _ptr(ts.who), N, B, ts.H, _ptr(ts.n_tok),
+                                       _ptr(ts.n_done), int(K), int(loss_kind),
+                                       int(accept_first), int(learner), float(eta), _ptr(state),
+                                       _ptr(weights), _ptr(selected), _ptr(played_loss),
+                                       _ptr(dev_status), _stream(stream)),
+           "hs_token_learner_step")
     return state, weights, selected

@@ -1,20 +1,11 @@
 // hs_learner.cu -- loss (Sec. 3.3), Hedge (App. B.1 remark) and NormalHedge
-// (App. D.6 figure) for B independent queries.
-//
-// One warp per query, lane i = drafter i (N <= 32), so every reduction over
-// drafters is a warp shuffle.  NormalHedge's scale is found by a warp-parallel
-// bisection: with x_i = [R_i]_+ / max R and kappa = (max R)^2 / (2c), the
-// scale equation becomes g(kappa) = (1/N) sum_i exp(kappa x_i^2) - e = 0 with
-// g increasing and the root in [1, 1 + ln N] (g(1) <= 0 since every term is
-// <= e; g(1 + ln N) >= 0 since the x = 1 term alone is N e).  Each round the
-// 32 lanes evaluate g at 32 interior points of the bracket and keep the
-// sub-interval where g changes sign, shrinking it 33-fold; 6 rounds take it
-// below fp32 resolution.  Then p_i is proportional to x_i exp(kappa x_i^2),
-// which equals ([R_i]_+/c) exp([R_i]_+^2 / 2c) up to the common factor.
+// (App. D.6 figure) for B independent queries: one warp per query, lane i =
+// drafter i (N <= 32); the round itself is hs_learner_core.cuh.
 #include <math.h>
 #include <stdint.h>
 
 #include "hs_common.cuh"
+#include "hs_learner_core.cuh"
 
 namespace hs {
 namespace {
@@ -42,18 +33,6 @@ struct LearnerArgs {
   int32_t* sel_out;       // [B]
   float* played;          // [B] or NULL: += f[sel_in]
 };
-
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
-  return v;
-}
-
-__device__ __forceinline__ float warp_min(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(kFull, v, o));
-  return v;
-}
 
 __global__ void __launch_bounds__(kWarpsPerBlock * 32) learner_kernel(LearnerArgs a) {
   pdl_wait();
@@ -87,61 +66,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) learner_kernel(LearnerArg
     if (lane == 0) a.played[b] += ok ? fs : __int_as_float(0x7fc00000);
   }
 
-  float w;
-  int sel;
-  if (a.learner == HS_HEDGE) {
-    // ---- Hedge: w = exp(-eta (L - min L)) / Z, choice = first argmin L ----
-    float L = act ? a.state_in[ib] : 0.f;
-    if (a.hedge_add_loss) L += f;
-    if (act && a.state_out) a.state_out[ib] = L;
-    const float Lmin = warp_min(act ? L : INFINITY);
-    const unsigned tie = __ballot_sync(kFull, act && L == Lmin);
-    sel = tie ? __ffs(tie) - 1 : 0;
-    w = act ? expf(-a.eta * (L - Lmin)) : 0.f;
-  } else {
-    // ---- NormalHedge steps 2-3: R_i += sum_j p_j (l_j - l_i) ----
-    const float p = act ? a.p_in[ib] : 0.f;
-    float inc = 0.f;
-    for (int j = 0; j < N; ++j) {
-      const float pj = __shfl_sync(kFull, p, j);
-      const float fj = __shfl_sync(kFull, f, j);
-      inc = fmaf(pj, fj - f, inc);
-    }
-    const float R = act ? a.state_in[ib] + inc : -INFINITY;
-    if (act && a.state_out) a.state_out[ib] = R;
-    const float Rmax = warp_max(R);
-    if (!(Rmax > 0.f)) {
-      // no positive regret: the scale equation has no root, p is uniform
-      w = act ? 1.f : 0.f;
-      sel = 0;
-    } else {
-      // ---- step 4 by warp-parallel bisection on kappa (see file header) ----
-      const float x = act ? fmaxf(R, 0.f) / Rmax : 0.f;
-      const float x2 = x * x;
-      float lo = 1.f, hi = 1.f + logf(float(N));
-      const float e1 = 2.71828182845904523536f;
-      for (int round = 0; round < 6; ++round) {
-        const float kap = lo + (hi - lo) * float(lane + 1) * (1.f / 33.f);
-        float g = 0.f;
-        for (int j = 0; j < N; ++j) g += expf(kap * __shfl_sync(kFull, x2, j));
-        const unsigned up = __ballot_sync(kFull, g >= e1 * float(N));
-        const int first = up ? __ffs(up) - 1 : 32;  // first point with g >= 0
-        const float klo = __shfl_sync(kFull, kap, first > 0 ? first - 1 : 0);
-        const float khi = __shfl_sync(kFull, kap, first < 32 ? first : 31);
-        if (first > 0) lo = klo;
-        if (first < 32) hi = khi;
-      }
-      const float kap = 0.5f * (lo + hi);
-      // ---- step 5: p_i proportional to x_i exp(kappa x_i^2) ----
-      w = act ? x * expf(kap * x2) : 0.f;
-      const unsigned top = __ballot_sync(kFull, act && R == Rmax);
-      sel = top ? __ffs(top) - 1 : 0;
-    }
-  }
-  float z = w;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(kFull, z, o);
-  if (act) a.weights_out[ib] = w / z;
+  float state = act ? a.state_in[ib] : 0.f;
+  float p = (act && a.learner == HS_NORMALHEDGE) ? a.p_in[ib] : 0.f;
+  const int sel = learner::round(a.learner, N, a.eta, f, a.hedge_add_loss != 0, state, p);
+  if (act && a.state_out) a.state_out[ib] = state;
+  if (act) a.weights_out[ib] = p;
   if (lane == 0) a.sel_out[b] = sel;
 }
 

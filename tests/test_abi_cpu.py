@@ -127,6 +127,37 @@ def test_learner_rejects_bad_arguments(hf):
     assert step(*bad) == hf.HS_ERR_INVALID_ARG
 
 
+def test_delayed_entries_reject_bad_arguments(hf):
+    lib = hf.lib()
+    E = hf
+    sample = [FAKE, 8, 4, FAKE, FAKE, None, None]
+    for idx, val, want in ((1, 0, E.HS_ERR_INVALID_ARG), (1, 33, E.HS_ERR_UNSUPPORTED),
+                           (3, None, E.HS_ERR_INVALID_ARG), (4, FAKE + 2, E.HS_ERR_MISALIGNED)):
+        bad = list(sample); bad[idx] = val
+        assert lib.hs_sample_select(*bad) == want, (idx, val)
+    chunk = [FAKE, FAKE, 8, 4, 6, E.HS_LOSS_LENGTH, E.HS_HEDGE, 0.5, FAKE, FAKE, None, FAKE, None,
+             None, None]
+    for idx, val, want in ((1, None, E.HS_ERR_INVALID_ARG), (4, 0, E.HS_ERR_INVALID_ARG),
+                           (5, 4, E.HS_ERR_INVALID_ARG), (7, -1.0, E.HS_ERR_INVALID_ARG),
+                           (1, FAKE + 1, E.HS_ERR_MISALIGNED), (2, 40, E.HS_ERR_UNSUPPORTED)):
+        bad = list(chunk); bad[idx] = val
+        assert lib.hs_chunk_learner_step(*bad) == want, (idx, val)
+    app = [FAKE, FAKE, 8, 4, 6, FAKE, FAKE, FAKE, 32, FAKE, FAKE, None, None]
+    for idx, val, want in ((8, 0, E.HS_ERR_INVALID_ARG), (9, None, E.HS_ERR_INVALID_ARG),
+                           (9, FAKE + 4, E.HS_ERR_MISALIGNED), (5, None, E.HS_ERR_INVALID_ARG),
+                           (2, 33, E.HS_ERR_UNSUPPORTED)):
+        bad = list(app); bad[idx] = val
+        assert lib.hs_token_append(*bad) == want, (idx, val)
+    tok = [FAKE, FAKE, 8, 4, 32, FAKE, FAKE, 8, E.HS_LOSS_LENGTH, 0, E.HS_NORMALHEDGE, 0.0, FAKE,
+           FAKE, FAKE, None, None, None]
+    for idx, val, want in ((7, 0, E.HS_ERR_INVALID_ARG), (7, 33, E.HS_ERR_INVALID_ARG),
+                           (9, -1, E.HS_ERR_INVALID_ARG), (8, 2, E.HS_ERR_INVALID_ARG),
+                           (10, 2, E.HS_ERR_INVALID_ARG), (6, FAKE + 4, E.HS_ERR_MISALIGNED),
+                           (12, None, E.HS_ERR_INVALID_ARG)):
+        bad = list(tok); bad[idx] = val
+        assert lib.hs_token_learner_step(*bad) == want, (idx, val)
+
+
 def test_binding_refuses_cpu_tensors(hf):
     import torch
     t = torch.zeros(1, 3, 8)
