@@ -61,6 +61,8 @@ def _bind(lib):
         "orc_token_loss": ([P, L, I, I], D),
         "orc_token_revealed": ([L, I, I, L], L),
         "orc_token_session": ([P, P, I, I, I, I, I, I, L, I, D, P, P, P, P, P, P], I),
+        "orc_learner_apply": ([P, I, I, I, I, D, P, P, P], I),
+        "orc_schedule_next": ([I, I, I, I, P, I, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -312,6 +314,36 @@ class Oracle:
         if st != OK:
             raise ValueError(f"oracle token_session rejected its arguments (status {st})")
         return state, weights, sel, played, done
+
+
+    # ---- App. B.5 practical heuristics --------------------------------------
+
+    def learner_apply(self, lv, learner_kind: int, eta: float, state, weights, selected):
+        """QFI-D catch-up over loss vectors lv [C,N,B] in order; new arrays."""
+        lv = _f64(lv)
+        C, N, B = lv.shape
+        state, weights = _f64(state).copy(), _f64(weights).copy()
+        sel = np.ascontiguousarray(selected, dtype=np.int32).copy()
+        st = self.lib.orc_learner_apply(_ptr(lv), C, N, B, int(learner_kind), float(eta),
+                                        _ptr(state), _ptr(weights), _ptr(sel))
+        if st != OK:
+            raise ValueError(f"oracle learner_apply rejected its arguments (status {st})")
+        return state, weights, sel
+
+    def schedule(self, warmup: int, batch_rounds: int, skip_tokens: int, hybrid_vectors: int,
+                 tokens):
+        """Decisions (evaluate, loss_kind, apply) for each round of a token
+        sequence tokens[r] (tokens generated by round r's chunk)."""
+        s = np.zeros(4, np.int64)
+        act = np.zeros(3, np.int32)
+        out = []
+        for t in tokens:
+            st = self.lib.orc_schedule_next(int(warmup), int(batch_rounds), int(skip_tokens),
+                                            int(hybrid_vectors), _ptr(s), int(t), _ptr(act))
+            if st != OK:
+                raise ValueError(f"oracle schedule rejected its arguments (status {st})")
+            out.append(tuple(int(x) for x in act))
+        return out
 
 
 _default: Oracle | None = None

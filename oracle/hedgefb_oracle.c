@@ -24,6 +24,8 @@
  *   - App. B.3:              chunk-level losses with the chunk horizon k_h
  *   - Sec. 3.2 (Fig. "Token-Level Game with Delay"): per-token losses and
  *                            the rule of when each is revealed
+ *   - App. B.5:              warm-up, skipped and batched updates, hybrid
+ *                            losses (a schedule), and a batch fed FIFO
  * Input logits are read as the very bytes the GPU reads: bf16 is widened by
  * a 16-bit shift, fp16 by its IEEE-754 binary16 definition, fp32 as is; all
  * three conversions to double are exact.
@@ -662,5 +664,83 @@ int orc_token_session(const double* alpha, const int* k_h, int H, int N, int B, 
   free(lv);
   free(st);
   free(wt);
+  return ORC_OK;
+}
+
+/* ---- App. B.5 practical heuristics: warm-up, batched and skipped updates,
+ * hybrid losses -------------------------------------------------------------- */
+
+/* QFI-D's catch-up over a batch of chunk-level loss vectors: the `count`
+ * vectors lv[c][N][B] are fed to Base in order (c = 0 first), one round each,
+ * for every query; state/weights/selected as in orc_learner_step. */
+int orc_learner_apply(const double* lv, int count, int N, int B, int learner_kind, double eta,
+                      double* state, double* weights, int* selected) {
+  if (N < 1 || B < 1 || count < 0) return ORC_BADARG;
+  double* one = (double*)malloc(sizeof(double) * (size_t)N);
+  double* st = (double*)malloc(sizeof(double) * (size_t)N);
+  double* wt = (double*)malloc(sizeof(double) * (size_t)N);
+  for (int b = 0; b < B; ++b) {
+    for (int i = 0; i < N; ++i) {
+      st[i] = state[i * B + b];
+      wt[i] = weights[i * B + b];
+    }
+    int choice = selected[b];
+    for (int c = 0; c < count; ++c) {
+      for (int i = 0; i < N; ++i) one[i] = lv[((size_t)c * N + i) * B + b];
+      base_update(learner_kind, eta, one, st, wt, N, &choice);
+    }
+    for (int i = 0; i < N; ++i) {
+      state[i * B + b] = st[i];
+      weights[i * B + b] = wt[i];
+    }
+    selected[b] = choice;
+  }
+  free(one);
+  free(st);
+  free(wt);
+  return ORC_OK;
+}
+
+/* The schedule of App. B.5, read as follows.  A round is one speculative
+ * chunk, after which the schedule decides:
+ *   - during the first warmup rounds: evaluate every drafter on the chunk
+ *     (panoramic feedback, one loss vector) and apply it at once (full
+ *     information every round);
+ *   - afterwards, "skipping updates by a fixed number of tokens": evaluate
+ *     only when at least skip_tokens tokens were generated since the last
+ *     evaluation (counting this chunk's), and "delayed batched feedback":
+ *     queue the vectors and apply the queue (FIFO, QFI-D) once every
+ *     batch_rounds rounds after the warm-up;
+ *   - "hybrid losses": the first hybrid_vectors loss vectors use the
+ *     acceptance-rate loss, later ones the length loss.
+ * State: s[0] rounds so far, s[1] tokens since the last evaluation, s[2]
+ * vectors made, s[3] vectors queued and not applied.  Outputs: act[0]
+ * evaluate, act[1] the loss kind of that vector, act[2] apply the queue
+ * (including this round's vector) before the next choice. */
+int orc_schedule_next(int warmup, int batch_rounds, int skip_tokens, int hybrid_vectors,
+                      int64_t* s, int tokens, int* act) {
+  if (warmup < 0 || batch_rounds < 1 || skip_tokens < 0 || hybrid_vectors < 0 || tokens < 0)
+    return ORC_BADARG;
+  const int64_t r = s[0];
+  int evaluate, apply;
+  if (r < warmup) {
+    evaluate = 1;
+    apply = 1;
+    s[1] = 0;
+  } else {
+    s[1] += tokens;
+    evaluate = s[1] >= skip_tokens;
+    if (evaluate) s[1] = 0;
+    apply = ((r - warmup + 1) % batch_rounds) == 0;
+  }
+  act[0] = evaluate;
+  act[1] = (evaluate && s[2] < hybrid_vectors) ? ORC_LOSS_ACCEPT : ORC_LOSS_LENGTH;
+  if (evaluate) {
+    s[2] += 1;
+    s[3] += 1;
+  }
+  act[2] = apply && s[3] > 0;
+  if (act[2]) s[3] = 0;
+  s[0] = r + 1;
   return ORC_OK;
 }

@@ -827,4 +827,75 @@ def check_token_session_unrevealed_is_unseen(o):
     assert sel2[3, 0] == sel[3, 0]
 
 
+# ---- App. B.5 practical heuristics ----------------------------------------------
+
+def check_schedule_hand_trace(o):
+    """warm-up 2, batch 3, skip 6 tokens, hybrid 2 vectors, worked by hand:
+    rounds 0-1 warm-up (evaluate, apply; the two acceptance-rate vectors);
+    then the token count since the last evaluation runs 7 (eval), 3, 6 (eval),
+    9 (eval), 1, 2, 10 (eval), 6 (eval), and the queue is applied at rounds
+    4 and 7 (every 3rd round after the warm-up; round 10 would be next)."""
+    got = o.schedule(2, 3, 6, 2, [5, 4, 7, 3, 3, 9, 1, 1, 8, 6])
+    A, Ln = orc.LOSS_ACCEPT, orc.LOSS_LENGTH
+    want = [(1, A, 1), (1, A, 1), (1, Ln, 0), (0, Ln, 0), (1, Ln, 1), (1, Ln, 0), (0, Ln, 0),
+            (0, Ln, 1), (1, Ln, 0), (1, Ln, 0)]
+    assert got == want, got
+
+
+def check_schedule_invariants(o):
+    """On random token counts: warm-up rounds evaluate and apply; later an
+    evaluation happens exactly when the tokens since the last one reach the
+    skip count; applies fall every batch_rounds rounds after the warm-up and
+    only with something queued; the first hybrid vectors are acceptance-rate
+    ones, all later ones length ones."""
+    rng = np.random.default_rng(68)
+    for _ in range(40):
+        W, Bt, S, Hy = (int(rng.integers(0, 8)), int(rng.integers(1, 14)),
+                        int(rng.integers(0, 15)), int(rng.integers(0, 10)))
+        toks = rng.integers(1, 10, 120)
+        dec = o.schedule(W, Bt, S, Hy, toks)
+        since, made, queued = 0, 0, 0
+        for r, (ev, kind, ap) in enumerate(dec):
+            if r < W:
+                assert ev == 1 and ap == 1
+                since = 0
+            else:
+                since += int(toks[r])
+                assert ev == (since >= S)
+                if ev:
+                    since = 0
+                assert ap == ((((r - W + 1) % Bt) == 0) and (queued + ev) > 0)
+            if ev:
+                assert kind == (orc.LOSS_ACCEPT if made < Hy else orc.LOSS_LENGTH)
+                made += 1
+                queued += 1
+            if ap:
+                queued = 0
+
+
+def check_learner_apply_batches(o):
+    """A batch fed through QFI-D: Hedge ends at the plain sum of the vectors
+    (and Hedge's closed form of it); NormalHedge equals one NormalHedge round
+    per vector in queue order; an empty batch changes nothing."""
+    rng = np.random.default_rng(69)
+    C, N, B = 7, 5, 4
+    lv = rng.random((C, N, B))
+    st0 = rng.random((N, B))
+    w0 = np.full((N, B), 1.0 / N)
+    s0 = rng.integers(0, N, B)
+    st, w, sel = o.learner_apply(lv, orc.HEDGE, 0.7, st0, w0, s0)
+    assert np.allclose(st, st0 + lv.sum(axis=0), rtol=0, atol=1e-12)
+    for b in range(B):
+        ww, ss = o.hedge(st[:, b], 0.7)
+        assert np.array_equal(w[:, b], ww) and sel[b] == ss
+    st, w, sel = o.learner_apply(lv, orc.NORMALHEDGE, 0.0, np.zeros((N, B)), w0, s0)
+    for b in range(B):
+        R, p = np.zeros(N), np.full(N, 1.0 / N)
+        for c in range(C):
+            R, p, ch, _ = o.normalhedge(R, lv[c, :, b], p)
+        assert np.array_equal(st[:, b], R) and np.array_equal(w[:, b], p) and sel[b] == ch
+    st, w, sel = o.learner_apply(lv[:0], orc.NORMALHEDGE, 0.0, st0, w0, s0)
+    assert np.array_equal(st, st0) and np.array_equal(w, w0) and np.array_equal(sel, s0)
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -81,6 +81,14 @@ MUTANTS = {
     "token_played_by_drafter_0": ("who[n] = choice;", "who[n] = 0;"),
     "qfid_hedge_not_cumulative": ("for (int i = 0; i < N; ++i) st[i] = st[i] + lv[i];",
                                   "for (int i = 0; i < N; ++i) st[i] = lv[i];"),
+    "apply_batch_reversed": ("for (int i = 0; i < N; ++i) one[i] = lv[((size_t)c * N + i) * B + b];",
+                             "for (int i = 0; i < N; ++i) one[i] = lv[((size_t)(count - 1 - c) * N + i) * B + b];"),
+    "schedule_skip_strict": ("evaluate = s[1] >= skip_tokens;", "evaluate = s[1] > skip_tokens;"),
+    "schedule_batch_off_by_one": ("apply = ((r - warmup + 1) % batch_rounds) == 0;",
+                                  "apply = ((r - warmup) % batch_rounds) == 0;"),
+    "schedule_hybrid_never": ("act[1] = (evaluate && s[2] < hybrid_vectors) ? ORC_LOSS_ACCEPT : ORC_LOSS_LENGTH;",
+                              "act[1] = ORC_LOSS_LENGTH;"),
+    "schedule_skip_keeps_count": ("    if (evaluate) s[1] = 0;\n", "\n"),
 }
 
 
