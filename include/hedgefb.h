@@ -314,6 +314,59 @@ hs_status hs_token_learner_step(const float* gamma_ring, const int32_t* who_ring
                                 int32_t* selected, float* played_loss, int* dev_status,
                                 void* stream);
 
+/* The chunk-level losses of hs_chunk_learner_step alone, without a learner
+ * update: loss_out [N,B] (device, fp32), e.g. one slot of a queue of delayed
+ * loss vectors for hs_learner_apply.  k_h as there (a query outside the range
+ * keeps its loss_out entries and sets *dev_status = HS_ERR_INVALID_ARG). */
+hs_status hs_chunk_losses(const float* alpha, const int32_t* k_h, int N, int B, int P,
+                          int loss_kind, float* loss_out, int* dev_status, void* stream);
+
+/* QFI-D's catch-up over a queue of chunk-level loss vectors (App. B.1; the
+ * batched feedback of App. B.5): vectors c = 0..count-1, in slots
+ * (first + c) mod Q of queue [Q,N,B] (device, fp32), are fed to the base
+ * learner in that order, one round each, for every query; state, weights
+ * and the choice as in hs_learner_step (selected[b] = the last round's
+ * choice).  0 <= first < Q, 0 <= count <= Q; count = 0 launches nothing. */
+hs_status hs_learner_apply(const float* queue, int Q, int first, int count, int N, int B,
+                           int learner, float eta, float* state, float* weights,
+                           int32_t* selected, void* stream);
+
+/* The practical schedule of App. B.5 ("skipping updates", batched delayed
+ * feedback, warm-up, "hybrid losses"), host only.  A round is one
+ * speculative chunk; after it hs_schedule_next decides, from the chunk's
+ * token count:
+ *   - in the first warmup_rounds rounds: evaluate every drafter on the
+ *     chunk and apply the vector at once (full information each round);
+ *   - afterwards: evaluate only when at least skip_tokens tokens were
+ *     generated since the last evaluation (this chunk's included); queue the
+ *     vectors, and apply the queue once every batch_rounds rounds counted
+ *     from the end of the warm-up (only when something is queued);
+ *   - the first hybrid_vectors vectors use HS_LOSS_ACCEPT, later ones
+ *     HS_LOSS_LENGTH.
+ * The paper's example setting is warmup 6, batch 12, skip 6. */
+typedef struct {
+  int warmup_rounds;
+  int batch_rounds;   /* >= 1 */
+  int skip_tokens;
+  int hybrid_vectors;
+} hs_schedule_config;
+
+typedef struct {      /* zero-initialise before the first round */
+  int64_t rounds;
+  int64_t tokens_since_eval;
+  int64_t vectors_made;
+  int64_t vectors_queued;
+} hs_schedule_state;
+
+typedef struct {
+  int evaluate;   /* 1: run the feedback on this chunk and queue its loss vector */
+  int loss_kind;  /* HS_LOSS_ACCEPT / HS_LOSS_LENGTH: that vector's loss */
+  int apply;      /* 1: feed the whole queue to the learner before the next choice */
+} hs_schedule_action;
+
+hs_status hs_schedule_next(const hs_schedule_config* cfg, hs_schedule_state* state,
+                           int tokens, hs_schedule_action* action);
+
 #ifdef __cplusplus
 }
 #endif

@@ -51,6 +51,9 @@ SIGNATURES = {
     "hs_token_append": ([_P, _P, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P], _I),
     "hs_token_learner_step": ([_P, _P, _I, _I, _I, _P, _P, _I, _I, _L, _I, _F, _P, _P, _P, _P,
                                _P, _P], _I),
+    "hs_chunk_losses": ([_P, _P, _I, _I, _I, _I, _P, _P, _P], _I),
+    "hs_learner_apply": ([_P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P], _I),
+    "hs_schedule_next": ([_P, _P, _I, _P], _I),
 }
 
 
@@ -390,3 +393,62 @@ def hs_token_learner_step(ts: TokenStream, K: int, loss_kind: int, learner: int,
                                        _ptr(dev_status), _stream(stream)),
            "hs_token_learner_step")
     return state, weights, selected
+
+
+def hs_chunk_losses(alpha: torch.Tensor, k_h: torch.Tensor, loss_kind: int, loss_out=None,
+                    dev_status=None, stream=None) -> torch.Tensor:
+    """Chunk-level loss vectors [N,B] with per-query chunk horizon k_h [B]."""
+    _need(alpha, "alpha", torch.float32)
+    N, B, P = alpha.shape
+    _need(k_h, "k_h", torch.int32, (B,))
+    if loss_out is None:
+        loss_out = torch.empty(N, B, dtype=torch.float32, device=alpha.device)
+    _need(loss_out, "loss_out", torch.float32, (N, B))
+    _check(lib().hs_chunk_losses(_ptr(alpha), _ptr(k_h), N, B, P, int(loss_kind), _ptr(loss_out),
+                                 _ptr(dev_status), _stream(stream)), "hs_chunk_losses")
+    return loss_out
+
+
+def hs_learner_apply(queue: torch.Tensor, first: int, count: int, learner: int, eta: float,
+                     state: torch.Tensor, weights: torch.Tensor, selected: torch.Tensor,
+                     stream=None):
+    """QFI-D catch-up over count loss vectors of queue [Q,N,B] from slot first."""
+    _need(queue, "queue", torch.float32)
+    Q, N, B = queue.shape
+    _need(state, "state", torch.float32, (N, B))
+    _need(weights, "weights", torch.float32, (N, B))
+    _need(selected, "selected", torch.int32, (B,))
+    _check(lib().hs_learner_apply(_ptr(queue), Q, int(first), int(count), N, B, int(learner),
+                                  float(eta), _ptr(state), _ptr(weights), _ptr(selected),
+                                  _stream(stream)), "hs_learner_apply")
+    return state, weights, selected
+
+
+class ScheduleConfig(ctypes.Structure):
+    _fields_ = [("warmup_rounds", ctypes.c_int), ("batch_rounds", ctypes.c_int),
+                ("skip_tokens", ctypes.c_int), ("hybrid_vectors", ctypes.c_int)]
+
+
+class ScheduleState(ctypes.Structure):
+    _fields_ = [("rounds", ctypes.c_int64), ("tokens_since_eval", ctypes.c_int64),
+                ("vectors_made", ctypes.c_int64), ("vectors_queued", ctypes.c_int64)]
+
+
+class ScheduleAction(ctypes.Structure):
+    _fields_ = [("evaluate", ctypes.c_int), ("loss_kind", ctypes.c_int), ("apply", ctypes.c_int)]
+
+
+class Schedule:
+    """App. B.5's practical schedule (host-side, in the library): one
+    next(tokens) per speculative chunk -> (evaluate, loss_kind, apply)."""
+
+    def __init__(self, warmup_rounds: int = 6, batch_rounds: int = 12, skip_tokens: int = 6,
+                 hybrid_vectors: int = 0):
+        self.cfg = ScheduleConfig(warmup_rounds, batch_rounds, skip_tokens, hybrid_vectors)
+        self.state = ScheduleState()
+
+    def next(self, tokens: int) -> tuple[int, int, int]:
+        act = ScheduleAction()
+        _check(lib().hs_schedule_next(ctypes.byref(self.cfg), ctypes.byref(self.state),
+                                      int(tokens), ctypes.byref(act)), "hs_schedule_next")
+        return act.evaluate, act.loss_kind, act.apply

@@ -4,7 +4,10 @@
 //                         inverse-CDF draw with a caller-supplied uniform,
 //                         one thread per query, fp32 sums in index order
 //   chunk_learner_kernel  chunk-level game with the chunk horizon k_h (App.
-//                         B.3): the losses use positions 1..k_h only
+//                         B.3): the losses use positions 1..k_h only; or the
+//                         losses alone, for a queue of delayed vectors
+//   apply_kernel          QFI-D catch-up over a queue of chunk-level loss
+//                         vectors (App. B.1; the batched feedback of B.5)
 //   token_append_kernel   the verified tokens of a chunk join each query's
 //                         token stream (a ring of gamma values)
 //   token_learner_kernel  QFI-D catch-up (App. B.1): every revealed token loss
@@ -83,6 +86,7 @@ struct ChunkArgs {
   int32_t* selected;     // [B]
   float* played;         // [B] or NULL
   int* dev_status;
+  int update;            // 0: write the losses only
 };
 
 __global__ void __launch_bounds__(kWarpsPerBlock * 32) chunk_learner_kernel(ChunkArgs a) {
@@ -116,6 +120,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) chunk_learner_kernel(Chun
     }
   }
   if (act && a.loss_out) a.loss_out[ib] = f;
+  if (!a.update) return;
   if (a.played) {
     const int s = a.selected[b];
     const bool ok = s >= 0 && s < a.N;
@@ -125,6 +130,39 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) chunk_learner_kernel(Chun
   float state = act ? a.state[ib] : 0.f;
   float p = (act && a.learner == HS_NORMALHEDGE) ? a.weights[ib] : 0.f;
   const int sel = learner::round(a.learner, a.N, a.eta, f, true, state, p);
+  if (act) {
+    a.state[ib] = state;
+    a.weights[ib] = p;
+  }
+  if (lane == 0) a.selected[b] = sel;
+}
+
+// ---- a queue of chunk-level loss vectors -----------------------------------------
+
+struct ApplyArgs {
+  const float* queue;    // [Q,N,B]: vector c sits in slot (first + c) mod Q
+  int Q, first, count, N, B, learner;
+  float eta;
+  float* state;          // [N,B]
+  float* weights;        // [N,B]
+  int32_t* selected;     // [B]
+};
+
+__global__ void __launch_bounds__(kWarpsPerBlock * 32) apply_kernel(ApplyArgs a) {
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int64_t b = int64_t(blockIdx.x) * kWarpsPerBlock + (threadIdx.x >> 5);
+  if (b >= a.B) return;  // whole warp
+  const bool act = lane < a.N;
+  const int64_t ib = int64_t(lane) * a.B + b;
+  float state = act ? a.state[ib] : 0.f;
+  float p = (act && a.learner == HS_NORMALHEDGE) ? a.weights[ib] : 0.f;
+  int sel = 0;
+  for (int c = 0; c < a.count; ++c) {  // FIFO
+    const int64_t slot = (int64_t(a.first) + c) % a.Q;
+    const float f = act ? a.queue[(slot * a.N + lane) * a.B + b] : 0.f;
+    sel = learner::round(a.learner, a.N, a.eta, f, true, state, p);
+  }
   if (act) {
     a.state[ib] = state;
     a.weights[ib] = p;
@@ -271,7 +309,7 @@ extern "C" hs_status hs_chunk_learner_step(const float* alpha, const int32_t* k_
       !hs::aligned(played_loss, 4) || !hs::aligned(dev_status, 4))
     return HS_ERR_MISALIGNED;
   hs::ChunkArgs a = {alpha, k_h, N, B, P, loss_kind, learner, eta, state, weights, loss_out,
-                     selected, played_loss, dev_status};
+                     selected, played_loss, dev_status, 1};
   if (hs::launch_pdl(hs::chunk_learner_kernel, dim3(hs::warp_blocks(B)),
                      dim3(hs::kWarpsPerBlock * 32), 0, static_cast<cudaStream_t>(stream),
                      a) != cudaSuccess)
@@ -360,5 +398,76 @@ extern "C" hs_status hs_token_learner_step(const float* gamma_ring, const int32_
                      dim3(hs::kWarpsPerBlock * 32), 0, static_cast<cudaStream_t>(stream),
                      a) != cudaSuccess)
     return HS_ERR_CUDA;
+  return HS_OK;
+}
+
+extern "C" hs_status hs_chunk_losses(const float* alpha, const int32_t* k_h, int N, int B, int P,
+                                     int loss_kind, float* loss_out, int* dev_status,
+                                     void* stream) {
+  if (N < 1 || B < 1 || P < 1 || int64_t(N) * B * P >= (int64_t(1) << 40))
+    return HS_ERR_INVALID_ARG;
+  if (N > HS_MAX_LEARNER_N) return HS_ERR_UNSUPPORTED;
+  if (loss_kind != HS_LOSS_LENGTH && loss_kind != HS_LOSS_ACCEPT) return HS_ERR_INVALID_ARG;
+  if (!alpha || !k_h || !loss_out) return HS_ERR_INVALID_ARG;
+  if (!hs::aligned(alpha, 4) || !hs::aligned(k_h, 4) || !hs::aligned(loss_out, 4) ||
+      !hs::aligned(dev_status, 4))
+    return HS_ERR_MISALIGNED;
+  hs::ChunkArgs a = {alpha, k_h, N, B, P, loss_kind, HS_HEDGE, 0.f, nullptr, nullptr, loss_out,
+                     nullptr, nullptr, dev_status, 0};
+  if (hs::launch_pdl(hs::chunk_learner_kernel, dim3(hs::warp_blocks(B)),
+                     dim3(hs::kWarpsPerBlock * 32), 0, static_cast<cudaStream_t>(stream),
+                     a) != cudaSuccess)
+    return HS_ERR_CUDA;
+  return HS_OK;
+}
+
+extern "C" hs_status hs_learner_apply(const float* queue, int Q, int first, int count, int N,
+                                      int B, int learner, float eta, float* state,
+                                      float* weights, int32_t* selected, void* stream) {
+  hs_status st = hs::check_nb(N, B);
+  if (st != HS_OK) return st;
+  if (Q < 1 || first < 0 || first >= Q || count < 0 || count > Q) return HS_ERR_INVALID_ARG;
+  if (learner != HS_HEDGE && learner != HS_NORMALHEDGE) return HS_ERR_INVALID_ARG;
+  if (!queue || !state || !weights || !selected) return HS_ERR_INVALID_ARG;
+  if (learner == HS_HEDGE && !(isfinite(eta) && eta >= 0.f)) return HS_ERR_INVALID_ARG;
+  if (!hs::aligned(queue, 4) || !hs::aligned(state, 4) || !hs::aligned(weights, 4) ||
+      !hs::aligned(selected, 4))
+    return HS_ERR_MISALIGNED;
+  if (count == 0) return HS_OK;  // QFI-D with an empty queue: nothing to do
+  hs::ApplyArgs a = {queue, Q, first, count, N, B, learner, eta, state, weights, selected};
+  if (hs::launch_pdl(hs::apply_kernel, dim3(hs::warp_blocks(B)), dim3(hs::kWarpsPerBlock * 32),
+                     0, static_cast<cudaStream_t>(stream), a) != cudaSuccess)
+    return HS_ERR_CUDA;
+  return HS_OK;
+}
+
+// App. B.5's schedule (host only; see the header for the reading).
+extern "C" hs_status hs_schedule_next(const hs_schedule_config* cfg, hs_schedule_state* st,
+                                      int tokens, hs_schedule_action* act) {
+  if (!cfg || !st || !act) return HS_ERR_INVALID_ARG;
+  if (cfg->warmup_rounds < 0 || cfg->batch_rounds < 1 || cfg->skip_tokens < 0 ||
+      cfg->hybrid_vectors < 0 || tokens < 0)
+    return HS_ERR_INVALID_ARG;
+  const int64_t r = st->rounds;
+  bool evaluate, apply;
+  if (r < cfg->warmup_rounds) {  // full information every round
+    evaluate = apply = true;
+    st->tokens_since_eval = 0;
+  } else {
+    st->tokens_since_eval += tokens;
+    evaluate = st->tokens_since_eval >= cfg->skip_tokens;
+    if (evaluate) st->tokens_since_eval = 0;
+    apply = (r - cfg->warmup_rounds + 1) % cfg->batch_rounds == 0;
+  }
+  act->evaluate = evaluate ? 1 : 0;
+  act->loss_kind =
+      (evaluate && st->vectors_made < cfg->hybrid_vectors) ? HS_LOSS_ACCEPT : HS_LOSS_LENGTH;
+  if (evaluate) {
+    ++st->vectors_made;
+    ++st->vectors_queued;
+  }
+  act->apply = (apply && st->vectors_queued > 0) ? 1 : 0;
+  if (act->apply) st->vectors_queued = 0;
+  st->rounds = r + 1;
   return HS_OK;
 }

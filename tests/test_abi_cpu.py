@@ -158,6 +158,31 @@ def test_delayed_entries_reject_bad_arguments(hf):
         assert lib.hs_token_learner_step(*bad) == want, (idx, val)
 
 
+def test_schedule_matches_oracle(hf):
+    """hs_schedule_next is host code: its decisions equal the oracle's on
+    random token counts and settings, including the paper's example."""
+    import numpy as np
+
+    import oracle
+    o = oracle.get()
+    rng = np.random.default_rng(5)
+    settings = [(6, 12, 6, 3)] + [(int(rng.integers(0, 9)), int(rng.integers(1, 15)),
+                                   int(rng.integers(0, 16)), int(rng.integers(0, 12)))
+                                  for _ in range(30)]
+    for cfg in settings:
+        toks = rng.integers(0, 10, 200)
+        sch = hf.Schedule(*cfg)
+        assert [sch.next(int(t)) for t in toks] == o.schedule(*cfg, toks), cfg
+
+
+def test_schedule_rejects_bad_settings(hf):
+    for cfg in ((6, 0, 6, 0), (-1, 12, 6, 0), (6, 12, -2, 0), (6, 12, 6, -1)):
+        with pytest.raises(hf.HedgeFBError):
+            hf.Schedule(*cfg).next(5)
+    with pytest.raises(hf.HedgeFBError):
+        hf.Schedule().next(-1)
+
+
 def test_binding_refuses_cpu_tensors(hf):
     import torch
     t = torch.zeros(1, 3, 8)

@@ -183,3 +183,50 @@ def test_token_ring_overflow_is_refused():
     hf.hs_token_append(ts, alpha, k_h, sel, dev_status=status)
     assert int(status.item()) == hf.HS_ERR_UNSUPPORTED
     assert ts.n_tok.cpu().tolist() == [5, 5]
+
+
+@pytest.mark.parametrize("learner", [hf.HS_HEDGE, hf.HS_NORMALHEDGE])
+def test_scheduled_session_matches_oracle(learner):
+    """App. B.5: the paper's example schedule (warm-up 6, batch 12, skip 6
+    tokens) with 3 hybrid vectors drives the losses-only kernel into a device
+    queue and the FIFO catch-up kernel; decisions, weights and choices after
+    every applied batch match the oracle's schedule and learner."""
+    rng = np.random.default_rng(4)
+    o = oracle.get()
+    R, N, B, P, Q, eta = 80, 8, 32, 9, 64, 0.25
+    cfg = (6, 12, 6, 3)
+    sch = hf.Schedule(*cfg)
+    ks = rng.integers(0, P, R)
+    dec = o.schedule(*cfg, ks + 1)
+    queue = torch.zeros(Q, N, B, device=DEV)
+    state = torch.zeros(N, B, device=DEV)
+    w = torch.full((N, B), 1.0 / N, device=DEV)
+    sel = torch.zeros(B, dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    o_state, o_w, o_sel = np.zeros((N, B)), np.full((N, B), 1.0 / N), np.zeros(B, np.int32)
+    pending, head, tail, applies = [], 0, 0, 0
+    for r in range(R):
+        ev, kind, ap = sch.next(int(ks[r]) + 1)
+        assert (ev, kind, ap) == dec[r], r
+        alpha = rng.random((N, B, P)).astype(np.float32)
+        if ev:
+            k_h = torch.full((B,), int(ks[r]), dtype=torch.int32, device=DEV)
+            hf.hs_chunk_losses(torch.from_numpy(alpha).to(DEV), k_h, kind,
+                               loss_out=queue[tail % Q], dev_status=status)
+            lv = np.array([[o.chunk_loss(alpha[i, b], int(ks[r]), kind) for b in range(B)]
+                           for i in range(N)])
+            assert_rel(to_np(queue[tail % Q]), lv, 1e-5, f"losses round {r}", atol=1e-6)
+            pending.append(lv)
+            tail += 1
+        if ap:
+            hf.hs_learner_apply(queue, head % Q, tail - head, learner, eta, state, w, sel)
+            o_state, o_w, o_sel = o.learner_apply(np.stack(pending), learner, eta, o_state, o_w,
+                                                  o_sel)
+            pending, head = [], tail
+            applies += 1
+            assert_rel(to_np(w), o_w, RTOL_WEIGHTS, f"weights after round {r}", atol=1e-6)
+            gs = sel.cpu().numpy()
+            for b in np.flatnonzero(gs != o_sel):
+                assert _near_tie(o_state, o_w, learner, gs[b], o_sel[b], b), (r, b)
+            o_sel = gs.copy()
+    assert applies >= 8 and int(status.item()) == hf.HS_OK
