@@ -7,11 +7,15 @@ the next choice) on one batch of seeded synthetic logits already resident in
 HBM.  Prints ONE JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
-                  [--mode stochastic|greedy|topl] [--branch-l L]
+                  [--mode stochastic|greedy|topl|token] [--branch-l L]
                   [--impl ours|reference]
 
 --mode topl runs the draft-tree feedback (Thm 2: the drafter proposes its L
 most likely tokens as a node's children) with a stochastic target.
+--mode token runs the stochastic feedback and then the token-level game with
+delay through QFI-D: the chunk's verified tokens join the per-query stream,
+the learner consumes every revealed token loss in token order, and the next
+drafter is drawn from the weights with a caller-supplied uniform.
 
 Timing: the K steps run as CUDA-graph replays on one stream, bracketed by
 CUDA events after a barrier + synchronize; inputs rotate over enough buffer
@@ -51,7 +55,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=5000)
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    ap.add_argument("--mode", choices=("stochastic", "greedy", "topl"), default="stochastic")
+    ap.add_argument("--mode", choices=("stochastic", "greedy", "topl", "token"),
+                    default="stochastic")
     ap.add_argument("--branch-l", type=int, default=10,
                     help="children per node of the draft tree (--mode topl)")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
@@ -145,6 +150,8 @@ KERNEL_SOURCES = {
                    "hs_stream.cu", "hs_stream.h"),
     "greedy": ("hs_common.cuh", "hs_feedback.cu", "hs_greedy.cu", "hs_greedy.h"),
     "topl": ("hs_common.cuh", "hs_feedback.cu", "hs_topl.cu", "hs_topl.h"),
+    "token": ("hs_common.cuh", "hs_feedback.cu", "hs_fused.cu", "hs_fused.h", "hs_stream.cu",
+              "hs_stream.h", "hs_delayed.cu", "hs_learner_core.cuh"),
 }
 
 
@@ -238,6 +245,7 @@ def run_ours(args):
     w = synth.WORKLOADS[args.workload]
     greedy = args.mode == "greedy"
     topl = args.mode == "topl"
+    token = args.mode == "token"
     learner = hf.HS_HEDGE if w.learner == "hedge" else hf.HS_NORMALHEDGE
     N, B, P, V = w.N, w.B, w.P, w.V
     props = torch.cuda.get_device_properties(dev)
@@ -245,6 +253,10 @@ def run_ours(args):
     n_sets = max(2, math.ceil(2 * l2 / w.bytes_per_call))
     sets = [synth.make_inputs(w, rnd=s, device=dev, seed=hdist.rank_seed(w.seed_base, rank) + s)
             for s in range(n_sets)]
+    if token:  # the uniforms of the sampled play are inputs, drawn per input set
+        gen = torch.Generator(device=dev).manual_seed(hdist.rank_seed(w.seed_base, rank) + 99)
+        for d in sets:
+            d["uniforms"] = torch.rand(w.B, generator=gen, device=dev)
 
     stream = torch.cuda.Stream(device=dev)
     alpha = torch.empty(N, B, P, device=dev)
@@ -257,6 +269,12 @@ def run_ours(args):
     weights = torch.full((N, B), 1.0 / N, device=dev)
     sel = torch.zeros(B, dtype=torch.int32, device=dev)
     eta = w.eta if w.eta else math.sqrt(8 * math.log(max(N, 2)) / 2000)
+    if token:
+        K = P - 1
+        ts = hf.TokenStream(N, B, K + 2 * P, dev)
+        k_full = torch.full((B,), K, dtype=torch.int32, device=dev)  # no censoring: fixed K
+        sel_arg = torch.zeros(B, dtype=torch.int32, device=dev)
+        played = torch.zeros(B, device=dev)
 
     def feedback(d):
         if topl and "path" in d:
@@ -275,10 +293,22 @@ def run_ours(args):
             hf.hs_feedback(d["target"], d["drafter"], w.temperature, greedy, alpha=alpha,
                            e_len=e_len, workspace=ws, dev_status=status, stream=stream)
 
+    def token_learner(d):
+        # this chunk's verified tokens (played by sel) join the stream; QFI-D
+        # catch-up on every revealed token loss; the next drafter is drawn
+        hf.hs_token_append(ts, alpha, k_full, sel, dev_status=status, stream=stream)
+        hf.hs_token_learner_step(ts, K, hf.HS_LOSS_LENGTH, learner, eta, state, weights, sel_arg,
+                                 played_loss=played, dev_status=status, stream=stream)
+        hf.hs_sample_select(weights, d["uniforms"], selected=sel, dev_status=status,
+                            stream=stream)
+
     def step(d):
         feedback(d)
-        hf.hs_learner_step(alpha, e_len, hf.HS_LOSS_LENGTH, learner, eta, state, weights, sel,
-                           stream=stream)
+        if token:
+            token_learner(d)
+        else:
+            hf.hs_learner_step(alpha, e_len, hf.HS_LOSS_LENGTH, learner, eta, state, weights,
+                               sel, stream=stream)
 
     # eager warm-up, then graphs of whole steps and of feedback calls
     with torch.cuda.stream(stream):
@@ -322,6 +352,7 @@ def run_ours(args):
     t_step = timed(step, args.steps)
     clk = clocks.stop()
     t_fb = timed(feedback, args.steps)
+    t_learn = timed(token_learner, args.steps) if token else None
     assert int(status.item()) == 0, hf.hs_status_string(int(status.item()))
 
     # ---- end to end through the public API from pinned host buffers ----
@@ -354,13 +385,16 @@ def run_ours(args):
     t_step = hdist.max_over_ranks(t_step, world, dev)
     t_fb = hdist.max_over_ranks(t_fb, world, dev)
     t_e2e = hdist.max_over_ranks(t_e2e, world, dev)
+    if token:
+        t_learn = hdist.max_over_ranks(t_learn, world, dev)
     evals_step = w.evals
     value = world * args.steps * evals_step / t_step
     peak, peak_src = measured_hbm_peak()
     fb_avg = t_fb / args.steps
     achieved = w.bytes_per_call / fb_avg / 1e9
-    launches_step = 1 + (hf.hs_feedback_topl_kernel_count(N, B, P, V) if topl else
-                         hf.hs_feedback_kernel_count(N, B, P, V, synth.DTYPES[w.dtype], greedy))
+    launches_step = (3 if token else 1) + (
+        hf.hs_feedback_topl_kernel_count(N, B, P, V) if topl else
+        hf.hs_feedback_kernel_count(N, B, P, V, synth.DTYPES[w.dtype], greedy))
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -392,6 +426,10 @@ def run_ours(args):
             "gpu_launches": launches_step * args.steps,
             "clocks": clk,
         }
+        if token:
+            line["config"]["learner_path"] = ("token-level game with delay through QFI-D, "
+                                              "length loss, K = P-1, sampled play")
+            line["learner_us_per_step"] = 1e6 * t_learn / args.steps
         print(json.dumps(line), flush=True)
     hdist.finalize(world)
 
