@@ -244,22 +244,35 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) token_learner_kernel(Toke
   const float* g = a.gamma + int64_t(b) * a.H * a.N + lane;
   float own = 0.f;
   int sel = 0;
-  for (; d < ready; ++d) {  // FIFO: token order
+  int slot = int(d % a.H);  // ring slot of token d
+  for (; d < ready; ++d, slot = slot + 1 == a.H ? 0 : slot + 1) {  // FIFO: token order
     float f = 0.f;
     if (act) {
       if (d < a.accept_first || a.loss_kind == HS_LOSS_ACCEPT) {
-        f = 1.f - g[(d % a.H) * a.N];
+        f = 1.f - g[int64_t(slot) * a.N];
       } else {
-        // Thm 3 for a K-token draft starting at token d
+        // Thm 3 for a K-token draft starting at token d; the window's loads
+        // are issued 8 at a time (slots wrap once at most: K <= H)
         float e = 1.f, prod = 1.f;
-        for (int j = 0; j < a.K; ++j) {
-          prod *= g[((d + j) % a.H) * a.N];
-          e += prod;
+        for (int j0 = 0; j0 < a.K; j0 += 8) {
+          float v[8];
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj) {
+            int sj = slot + j0 + jj;
+            sj -= sj >= a.H ? a.H : 0;
+            v[jj] = j0 + jj < a.K ? g[int64_t(sj) * a.N] : 1.f;
+          }
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj)
+            if (j0 + jj < a.K) {
+              prod *= v[jj];
+              e += prod;
+            }
         }
         f = 1.f - e / float(a.K + 1);
       }
     }
-    const int pl = a.who[int64_t(b) * a.H + d % a.H];
+    const int pl = a.who[int64_t(b) * a.H + slot];
     own += __shfl_sync(kFull, f, pl >= 0 && pl < a.N ? pl : 0);
     sel = learner::round(a.learner, a.N, a.eta, f, true, state, p);
   }

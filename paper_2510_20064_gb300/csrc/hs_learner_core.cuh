@@ -9,8 +9,11 @@
 // root in [1, 1 + ln N] (g(1) <= 0 since every term is <= e; g(1 + ln N) >= 0
 // since the x = 1 term alone is N e).  Each round the 32 lanes evaluate g at
 // 32 interior points of the bracket and keep the sub-interval where g changes
-// sign, shrinking it 33-fold; 6 rounds take it below fp32 resolution.  Then
-// p_i is proportional to x_i exp(kappa x_i^2), which equals
+// sign, shrinking it 33-fold; 6 rounds take it below fp32 resolution.  The
+// terms exp(kappa x_j^2) of g are formed as 2^{kappa y_j}, y_j = x_j^2 log2(e),
+// with the hardware exp2 (about 2^-22 relative), and the drafters beyond N
+// carry y = -inf, so they add exact zeros and the sums run over whole groups
+// of 8 lanes.  Then p_i is proportional to x_i exp(kappa x_i^2), which equals
 // ([R_i]_+/c) exp([R_i]_+^2 / 2c) up to the common factor.
 #pragma once
 
@@ -60,12 +63,17 @@ __device__ __forceinline__ int round(int learner, int N, float eta, float f, boo
     w = act ? expf(-eta * (L - Lmin)) : 0.f;
   } else {
     // ---- NormalHedge steps 2-3: R_i += sum_j p_j (l_j - l_i) ----
+    // (lanes >= N hold p = 0 and f = 0, so their terms are exact zeros)
     const float pi = act ? p : 0.f;
+    const float fi = act ? f : 0.f;
     float inc = 0.f;
-    for (int j = 0; j < N; ++j) {
-      const float pj = __shfl_sync(kFull, pi, j);
-      const float fj = __shfl_sync(kFull, f, j);
-      inc = fmaf(pj, fj - f, inc);
+    for (int j0 = 0; j0 < N; j0 += 8) {
+#pragma unroll
+      for (int jj = 0; jj < 8; ++jj) {
+        const float pj = __shfl_sync(kFull, pi, j0 + jj);
+        const float fj = __shfl_sync(kFull, fi, j0 + jj);
+        inc = fmaf(pj, fj - fi, inc);
+      }
     }
     const float R = act ? state + inc : -INFINITY;
     state = R;
@@ -78,12 +86,16 @@ __device__ __forceinline__ int round(int learner, int N, float eta, float f, boo
       // ---- step 4 by warp-parallel bisection on kappa (see file header) ----
       const float x = act ? fmaxf(R, 0.f) / Rmax : 0.f;
       const float x2 = x * x;
+      const float y = act ? x2 * kLog2e : -INFINITY;
       float lo = 1.f, hi = 1.f + logf(float(N));
       const float e1 = 2.71828182845904523536f;
       for (int r = 0; r < 6; ++r) {
         const float kap = lo + (hi - lo) * float(lane + 1) * (1.f / 33.f);
         float g = 0.f;
-        for (int j = 0; j < N; ++j) g += expf(kap * __shfl_sync(kFull, x2, j));
+        for (int j0 = 0; j0 < N; j0 += 8) {
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj) g += ex2(kap * __shfl_sync(kFull, y, j0 + jj));
+        }
         const unsigned up = __ballot_sync(kFull, g >= e1 * float(N));
         const int first = up ? __ffs(up) - 1 : 32;  // first point with g >= 0
         const float klo = __shfl_sync(kFull, kap, first > 0 ? first - 1 : 0);
