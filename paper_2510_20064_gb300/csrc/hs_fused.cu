@@ -50,6 +50,14 @@ constexpr int kXArm = 4;    // the xbar phase of row g + kXArm is armed at row g
 constexpr int kASlots = 8;  // tiles whose alpha partials may be in flight (rank 0)
 constexpr int kTSlots = 4;  // tiles whose per-warp partials await the coordinator
 constexpr int kMaxU = 5;    // 16-byte vectors per consumer thread and row
+
+// TMEM row slots of exponentials per consumer thread: the 512 columns of a
+// lane quadrant hold, for each of its 4 consumer warps, the tile's p and the
+// slots, 8U columns each.  (Three slots fit when U <= 4, for rows pipelined
+// four deep; measured, that was no faster: the row rate is not set by the
+// exchange latency the depth would hide.)
+constexpr int kSlots = 2;
+constexpr int kMaxRanks = 16;  // CTAs per cluster (above 8: a non-portable size)
 constexpr long long kTimeoutCycles = 1LL << 31;  // about a second
 constexpr uint32_t kNegInfBf16x2 = 0xFF80FF80u;
 constexpr uint32_t kNegInfF16x2 = 0xFC00FC00u;
@@ -61,13 +69,13 @@ struct __align__(16) Shared {
   uint64_t accbar[kTSlots];        // every consumer warp posted a tile's partials
   uint64_t abar[kASlots];          // every rank's tile partials arrived (rank 0)
   float2 red[kXSlots][16];                // per-warp (offset, sum) of a row
-  float2 xch[kXSlots][kMaxC];             // per-rank (offset, sum) of a row
+  float2 xch[kXSlots][kMaxRanks];         // per-rank (offset, sum) of a row
   float acc[kTSlots][kMaxN][kConsumerWarps];  // per-warp alpha partials of a tile
   uint64_t rowbar[kXSlots];               // a row's per-warp scales are published
   float rowf[kXSlots][16];                // per-warp scale f: p or q = f * exponential
   uint32_t tval[kASlots];                 // tile's target row is usable
   uint32_t dval[kASlots];                 // bit i: tile's drafter i row is usable
-  float clacc[kASlots][kMaxC][kMaxN];     // per-rank alpha partials (rank 0)
+  float clacc[kASlots][kMaxRanks][kMaxN];  // per-rank alpha partials (rank 0)
   int error;
   uint32_t tmem_base;  // tensor memory: p and two rows of exponentials per thread
 };
@@ -387,7 +395,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
   constexpr uint32_t stage_bytes = SU * 2;
   // TMEM: the consumer warps of one lane quadrant (warps w, w+4, ...) each
   // take 3 * 8U columns (p and two row slots) of the 512
-  static_assert(((kConsumerWarps + 3) / 4) * 3 * U * 8 <= 512, "TMEM columns");
+  constexpr int kDepth = kSlots + 1;  // rows in flight per consumer warp
+  static_assert(((kConsumerWarps + 3) / 4) * (1 + kSlots) * U * 8 <= 512, "TMEM columns");
+  static_assert(kDepth <= kXArm, "a row's exchange slot is re-armed kXArm rows later");
   unsigned char* ring = smem_raw + ((sizeof(Shared) + 127) & ~size_t(127));
 
   pdl_trigger();  // the small e_len kernel may take the SMs no cluster uses
@@ -491,16 +501,16 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       const int x = g % kXSlots;
       wait_local(saddr(&sh.xbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
       // every lane merges the C pairs itself, in rank order
-      float2 v[kMaxC];
+      float2 v[kMaxRanks];
 #pragma unroll
-      for (int rr = 0; rr < kMaxC; ++rr)
+      for (int rr = 0; rr < kMaxRanks; ++rr)
         v[rr] = rr < int(C) ? sh.xch[x][rr] : make_float2(-INFINITY, 0.f);
       float O = v[0].x;
 #pragma unroll
-      for (int rr = 1; rr < kMaxC; ++rr) O = fmax_nan(O, v[rr].x);
+      for (int rr = 1; rr < kMaxRanks; ++rr) O = fmax_nan(O, v[rr].x);
       float Z = 0.f;
 #pragma unroll
-      for (int rr = 0; rr < kMaxC; ++rr)
+      for (int rr = 0; rr < kMaxRanks; ++rr)
         Z += (v[rr].x == -INFINITY || O == -INFINITY) ? 0.f : v[rr].y * ex2(v[rr].x - O);
       const bool valid = isfinite(O) && Z > 0.f;
       if (lane < kConsumerWarps) {
@@ -531,7 +541,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
         issue(sh, ring + (g % kStages) * stage_bytes, g + kStages, walk.next(p, ncl, slice0),
               bytes);
       // row g - kXArm's exchange is complete here (the consumers have passed
-      // pass 2 of row g - 3), so its slot can be armed for row g + kXArm,
+      // pass 2 of row g - kDepth, kDepth <= kXArm), so its slot can be armed
+      // for row g + kXArm,
       // which no rank sends before this CTA has posted row g + 1
       if (lane == 0 && g + kXArm < G)
         mbar_arrive_tx(saddr(&sh.xbar[(g + kXArm) % kXSlots]), 8u * C);
@@ -543,7 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       if (lane < int(C))
         st_async_f2(mapa(saddr(&sh.xch[x][rank]), lane), oc, sc, mapa(saddr(&sh.xbar[x]), lane));
       if (g > 0) publish(g - 1);
-      while (reduced < my_tiles && (reduced + 1) * R + 2 <= g) reduce_tile(reduced++);
+      // a tile's alpha partials are complete once the consumers have passed
+      // pass 2 of its last row, kDepth rows behind the posts of row g
+      while (reduced < my_tiles && (reduced + 1) * R + kDepth - 1 <= g) reduce_tile(reduced++);
     }
     if (G > 0) publish(G - 1);
     while (reduced < my_tiles) reduce_tile(reduced++);
@@ -562,7 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
     // this thread's TMEM lane (the warp's quadrant) and columns: [0, 8U) p of
     // the tile's target, [8U (1+s), 8U (2+s)) the exponentials of row slot s
     const uint32_t tbase = sh.tmem_base + (uint32_t(32 * (warp & 3)) << 16) +
-                           uint32_t((warp >> 2) * 3 * U * 8);
+                           uint32_t((warp >> 2) * (1 + kSlots) * U * 8);
 
     // pass 1: load row g from the ring (then release the stage); warp max;
     // exponentials relative to the warp's offset; post the warp's (offset,
@@ -624,14 +637,14 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       }
     };
 
-    // pass 2 of row g (exponentials in TMEM slot g & 1): target -> p into
+    // pass 2 of row g (exponentials in TMEM slot g % kSlots): target -> p into
     // TMEM; drafter i -> alpha partial
     auto pass2 = [&](int g, int j, int r) {
       const int x = g % kXSlots;
       wait_local(saddr(&sh.rowbar[x]), uint32_t(g / kXSlots) & 1u, sh, p.dev_status);
       const float f = sh.rowf[x][warp];
       const f2_t ff = pk(f, f);
-      const uint32_t te = tbase + uint32_t((1 + (g & 1)) * U * 8);
+      const uint32_t te = tbase + uint32_t((1 + g % kSlots) * U * 8);
       tmem_wait_st();  // this row's exponentials and the tile's p have landed
       if (r == 0) {
 #pragma unroll
@@ -692,13 +705,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
       }
     };
 
-    // three rows in flight: pass 1 of row g+2 runs before pass 2 of row g,
-    // so the cluster exchange of a row has two rows of work to hide behind
+    // kDepth rows in flight: pass 1 of row g + kDepth - 1 runs before pass 2
+    // of row g, so the cluster exchange of a row has kDepth - 1 rows of work
+    // to hide behind; row r's exponentials live in TMEM slot r % kSlots (row
+    // g + kSlots takes the slot row g frees)
     f2_t E[U * 4];
     int jj = 0, rr = 0;  // tile and row within tile of row g
-    for (int g = -2; g < G; ++g) {
-      const bool more = g + 2 < G;
-      if (more) pass1(g + 2, E);
+    for (int g = -kSlots; g < G; ++g) {
+      const bool more = g + kSlots < G;
+      if (more) pass1(g + kSlots, E);
       if (g >= 0) {
         pass2(g, jj, rr);
         if (++rr == R) {
@@ -706,7 +721,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_kernel(const Params p) {
           ++jj;
         }
       }
-      if (more) store_row(g & 1, E);
+      if (more) store_row((g + kSlots) % kSlots, E);
     }
   }
   // no CTA may leave while a peer can still write into its shared memory;
@@ -737,34 +752,33 @@ struct Plan {
   int C = 0, S = 0, U = 0;
 };
 
-Plan plan_for(int V) {
+// The slice and vector count for clusters of C CTAs; C = 0 when a slice does
+// not fit a CTA.
+Plan plan_c(int V, int C) {
   Plan pl;
-  for (int C = 1; C <= kMaxC; C *= 2) {
-    const int S = ((V + C - 1) / C + 7) / 8 * 8;
-    const int U = (S + kConsumers * 8 - 1) / (kConsumers * 8);
-    if (U <= kMaxU && shared_bytes(U) <= kSmemLimit) {
-      pl.C = C;
-      pl.S = S;
-      pl.U = U;
-      return pl;
-    }
+  const int S = ((V + C - 1) / C + 7) / 8 * 8;
+  const int U = (S + kConsumers * 8 - 1) / (kConsumers * 8);
+  if (U <= kMaxU && shared_bytes(U) <= kSmemLimit) {
+    pl.C = C;
+    pl.S = S;
+    pl.U = U;
   }
   return pl;
 }
 
-template <int DT, int U>
-hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
-  auto kern = fused_kernel<DT, U>;
-  const size_t smem = shared_bytes(pl.U);
-  static int configured_smem = 0;  // attribute is per kernel; raise it once
-  if (configured_smem < int(smem)) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) !=
-        cudaSuccess)
-      return HS_ERR_CUDA;
-    configured_smem = int(smem);
+// The smallest portable cluster (1, 2, 4 or 8 CTAs) that holds a row.
+Plan plan_for(int V) {
+  for (int C = 1; C <= kMaxC; C *= 2) {
+    const Plan pl = plan_c(V, C);
+    if (pl.C) return pl;
   }
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[2];
+  return Plan();
+}
+
+template <int DT, int U>
+void fill_config(cudaLaunchConfig_t& cfg, cudaLaunchAttribute (&attr)[2], const Plan& pl,
+                 size_t smem, cudaStream_t stream) {
+  cfg = {};
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = pl.C;
   attr[0].val.clusterDim.y = 1;
@@ -777,21 +791,81 @@ hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cfg.gridDim = dim3(pl.C);
-  // resident clusters for this (cluster size, shared memory); queried once, on
-  // the first call, so that later calls can be captured into CUDA graphs
-  static int cached_c = 0, cached_smem = 0, max_clusters = 0;
-  if (cached_c != pl.C || cached_smem != int(smem)) {
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1)
-      return HS_ERR_UNSUPPORTED;
-    max_clusters = n;
-    cached_c = pl.C;
-    cached_smem = int(smem);
+}
+
+// Resident clusters of fused_kernel<DT, U> with clusters of pl.C CTAs (0 when
+// none fit).  Each cluster size is queried once, on the first call, so that
+// later calls can be captured into CUDA graphs; the kernel's attributes
+// (shared memory, non-portable cluster sizes) are raised once as well.
+template <int DT, int U>
+int resident_clusters(const Plan& pl) {
+  auto kern = fused_kernel<DT, U>;
+  const size_t smem = shared_bytes(U);
+  static bool configured = false;
+  if (!configured) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess)
+      return 0;
+    configured = true;
   }
+  static int resident[kMaxRanks + 1] = {};  // 0: not queried yet, -1: none fit
+  if (resident[pl.C] == 0) {
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[2];
+    fill_config<DT, U>(cfg, attr, pl, smem, nullptr);
+    int n = 0;
+    resident[pl.C] = (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0)
+                         ? n
+                         : -1;
+  }
+  return resident[pl.C] > 0 ? resident[pl.C] : 0;
+}
+
+template <int DT>
+int clusters_of(const Plan& pl) {
+  switch (pl.U) {
+    case 1: return resident_clusters<DT, 1>(pl);
+    case 2: return resident_clusters<DT, 2>(pl);
+    case 3: return resident_clusters<DT, 3>(pl);
+    case 4: return resident_clusters<DT, 4>(pl);
+    default: return resident_clusters<DT, 5>(pl);
+  }
+}
+
+// The cluster size, from the smallest one that holds a row up to 16 CTAs,
+// that keeps the most SMs busy (ties: the smaller).  On a GB300, clusters of
+// 8 CTAs fit 15 times (120 SMs), of 9 CTAs 15 times (135 SMs), of 10 CTAs 13
+// times; V = 151 936 and 128 256 take 9.
+template <int DT>
+Plan choose_plan(int V) {
+  Plan best = plan_for(V);
+  if (best.C == 0) return best;
+  int best_sms = best.C * clusters_of<DT>(best);
+  for (int C = best.C + 1; C <= kMaxRanks; ++C) {
+    const Plan pl = plan_c(V, C);
+    if (pl.C == 0) continue;
+    const int sms = C * clusters_of<DT>(pl);
+    if (sms > best_sms) {
+      best = pl;
+      best_sms = sms;
+    }
+  }
+  return best;
+}
+
+template <int DT, int U>
+hs_status launch_t(const Params& p, const Plan& pl, cudaStream_t stream) {
+  const int max_clusters = resident_clusters<DT, U>(pl);
+  if (max_clusters < 1) return HS_ERR_UNSUPPORTED;
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[2];
+  fill_config<DT, U>(cfg, attr, pl, shared_bytes(U), stream);
   const int nclusters = max(1, min(p.ntiles, max_clusters));
   cfg.gridDim = dim3(unsigned(nclusters * pl.C));
   cfg.numAttrs = 2;  // cluster shape + programmatic dependent launch
-  if (cudaLaunchKernelEx(&cfg, kern, p) != cudaSuccess) return HS_ERR_CUDA;
+  if (cudaLaunchKernelEx(&cfg, fused_kernel<DT, U>, p) != cudaSuccess) return HS_ERR_CUDA;
   return HS_OK;
 }
 
@@ -837,7 +911,8 @@ bool eligible(const void* target, const void* drafter, int dtype, int N, int V, 
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
                  int N, int B, int P, int V, float c, float* alpha, float* e_len,
                  int* dev_status, cudaStream_t stream) {
-  const Plan pl = plan_for(V);
+  const Plan pl = dtype == HS_BF16 ? choose_plan<HS_BF16>(V) : choose_plan<HS_FP16>(V);
+  if (pl.C == 0) return HS_ERR_UNSUPPORTED;
   Params p;
   p.target = target;
   p.path = path;
