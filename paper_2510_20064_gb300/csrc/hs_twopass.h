@@ -1,0 +1,26 @@
+// hs_twopass.h -- internal interface of the two-pass-per-CTA stochastic
+// kernel (hs_twopass.cu) the cluster kernel's dispatch hands some shapes to.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "hedgefb.h"
+
+namespace hs {
+namespace twopass {
+
+// Whether this kernel should take a call: the cluster kernel would leave
+// SMs idle (cluster_sms < sms), every SM gets at least two tiles, and the
+// rows each SM keeps in L2 between its two passes fit in 90% of L2.
+bool preferred(int V, int elem_bytes, int tiles, int sms, int cluster_sms, size_t l2_bytes);
+
+// alpha of tiles t0 .. B*P-1 (bf16/fp16, V % 8 == 0, 16-byte-aligned rows),
+// one CTA per tile at a time over `grid` CTAs (one per SM).
+hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
+                 int N, int B, int P, int V, float c, int t0, int grid, float* alpha,
+                 int* dev_status, cudaStream_t stream);
+
+}  // namespace twopass
+}  // namespace hs

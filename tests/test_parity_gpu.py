@@ -286,3 +286,34 @@ def test_streaming_kernel_many_tiles():
     col = oracle_alpha_rows(d, [(2, 7, k) for k in range(4)], 0.9, False)
     assert_rel(np.array([e[2, 7]]), np.array([1.0 + np.cumprod(col[:-1]).sum()]), RTOL_ALPHA,
                "streaming e_len")
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp16"])
+def test_two_pass_kernel_every_alpha(dtype):
+    """320 tiles of 76808-logit rows: the cluster kernel would hold them on 144
+    of the SMs and the rows of every SM fit in L2, so the two-pass kernel
+    takes the call (one CTA per SM, the second pass from L2); every alpha and
+    e_len is compared."""
+    w = synth.Workload("two_pass", N=2, B=80, P=4, V=76808, dtype=dtype, temperature=0.8,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=41)
+    compare_full(d, 0.8, False)
+
+
+def test_two_pass_kernel_flags_bad_rows():
+    """A NaN drafter row, and an out-of-range path node: only their alphas
+    are NaN, with the status the other kernels report."""
+    w = synth.Workload("two_pass", N=2, B=80, P=4, V=76808, dtype="bf16", temperature=1.0,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=42)
+    d["drafter"][1, 77, 3, 5] = float("nan")
+    a, e, st = run(d, 1.0, False)
+    ra, re, rst = oracle_feedback(d, 1.0, False)
+    assert st == hf.HS_ERR_NONFINITE
+    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 1
+    assert_rel(a, ra, RTOL_ALPHA, "alpha next to a NaN row")
+    t = synth.make_inputs(W["tree_path"], device=DEV, B=80, N=2, V=76808, seed=43)
+    t["path"][79, 2] = 999
+    a, e, st = run(t, 1.0, False)
+    assert st == hf.HS_ERR_INVALID_ARG
+    assert np.isnan(a[:, 79, 2]).all() and np.isnan(a).sum() == 2
