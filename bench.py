@@ -147,11 +147,12 @@ def measured_hbm_peak():
 # the sources of the kernels a feedback call of each mode launches
 KERNEL_SOURCES = {
     "stochastic": ("hs_common.cuh", "hs_feedback.cu", "hs_fused.cu", "hs_fused.h",
-                   "hs_stream.cu", "hs_stream.h"),
+                   "hs_stream.cu", "hs_stream.h", "hs_twopass.cu", "hs_twopass.h"),
     "greedy": ("hs_common.cuh", "hs_feedback.cu", "hs_greedy.cu", "hs_greedy.h"),
     "topl": ("hs_common.cuh", "hs_feedback.cu", "hs_topl.cu", "hs_topl.h"),
     "token": ("hs_common.cuh", "hs_feedback.cu", "hs_fused.cu", "hs_fused.h", "hs_stream.cu",
-              "hs_stream.h", "hs_delayed.cu", "hs_learner_core.cuh"),
+              "hs_stream.h", "hs_twopass.cu", "hs_twopass.h", "hs_delayed.cu",
+              "hs_learner_core.cuh"),
 }
 
 
