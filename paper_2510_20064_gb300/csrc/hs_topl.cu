@@ -626,9 +626,10 @@ __global__ void __launch_bounds__(kThreads) alpha_kernel(const Params p) {
 
 // Warps per row: enough that the GPU holds about kWarpTarget warps when rows
 // are few (at most 16, and never more parts than whole steps in the row).
-constexpr int64_t kWarpTarget = 2432;  // 152 SMs x 16 warps
+constexpr int64_t kFewRows = 1216;     // below this many rows a row is split
+constexpr int64_t kWarpTarget = 4864;  // 152 SMs x 32 warps: one full wave of topl_kernel
 int split_of(int64_t rows, int V) {
-  if (2 * rows > kWarpTarget) return 1;  // splitting adds insertions; only for few rows
+  if (rows > kFewRows) return 1;  // splitting adds insertions; only for few rows
   int64_t S = (kWarpTarget + rows - 1) / rows;
   const int64_t steps = (int64_t(V) + 32 * kUnroll * 8 - 1) / (32 * kUnroll * 8);
   if (S > steps) S = steps;
