@@ -5,10 +5,11 @@
 //                           max of the stored logits and the first index
 //                           holding it; every logit is read once, 8 16-byte
 //                           loads in flight per thread
-//   greedy_finalize_kernel  one warp per (drafter i, query b): combines the
-//                           chunk partials of the target and drafter rows in
-//                           chunk order (first index wins ties), compares,
-//                           and forms e_len from the P positions
+//   greedy_finalize_kernel  one warp per drafter row (i, b, k): combines the
+//                           chunk partials of its target and drafter rows in
+//                           chunk order (first index wins ties) and compares;
+//                           the last of the P warps of (i, b) to finish (an
+//                           atomic count the argmax kernel zeroes) forms e_len
 // All of it is exact: maxima and indices of the stored values.
 #include <math.h>
 #include <stdint.h>
@@ -35,8 +36,10 @@ template <int DT, bool VEC>
 __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int B, int P, int V, Part* __restrict__ parts,
-    int nchunk) {
+    int nchunk, int* __restrict__ counters, int ncounters) {
   pdl_wait();
+  if (counters && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int x = threadIdx.x; x < ncounters; x += kThreads) counters[x] = 0;
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kS = kUnroll * kV;
   __shared__ float red_m[kWarps];
@@ -101,40 +104,53 @@ __device__ __forceinline__ void combine(const Part* __restrict__ pr, int nchunk,
 __global__ void greedy_finalize_kernel(const Part* __restrict__ parts, int nchunk,
                                        const int32_t* __restrict__ path, int M, int N, int B,
                                        int P, float* __restrict__ alpha,
-                                       float* __restrict__ e_len, int* dev_status) {
+                                       float* __restrict__ e_len, int* __restrict__ counters,
+                                       int* dev_status) {
   pdl_wait();
-  const int64_t gw = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  if (gw >= int64_t(N) * B) return;  // whole warp
-  const int64_t i = gw / B, b = gw % B;
+  const int64_t r = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;  // row (i, b, k)
   const int64_t BP = int64_t(B) * P;
+  if (r >= int64_t(N) * BP) return;  // whole warp
   const int l = threadIdx.x & 31;
-  float e = 1.f, prod = 1.f;
-  int err = HS_OK;
-  for (int k = 0; k < P; ++k) {
-    const int64_t tile = b * P + k;
-    const int64_t drow = (i * B + b) * P + k;
-    float mt, md;
-    int at, ad;
-    combine(parts + tile * nchunk, nchunk, mt, at);
-    combine(parts + (BP + drow) * nchunk, nchunk, md, ad);
-    const bool bad_path = path && (path[tile] < 0 || path[tile] >= M);
+  const int64_t tile = r % BP;
+  float mt, md;
+  int at, ad;
+  combine(parts + tile * nchunk, nchunk, mt, at);
+  combine(parts + (BP + r) * nchunk, nchunk, md, ad);
+  const bool bad_path = path && (path[tile] < 0 || path[tile] >= M);
+  int last = 0;
+  if (l == 0) {
     float a;
     if (bad_path || !isfinite(mt) || !isfinite(md)) {
       a = __int_as_float(0x7fc00000);
-      if (err == HS_OK) err = bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE;
+      report(dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
     } else {
       a = (at == ad) ? 1.f : 0.f;
     }
-    if (l == 0) alpha[drow] = a;
-    if (k < P - 1) {
-      prod *= a;
-      e += prod;
+    alpha[r] = a;
+    if (e_len) {
+      __threadfence();  // alpha[r] before the count
+      last = atomicAdd(&counters[r / P], 1) == P - 1;
     }
   }
-  if (l == 0) {
-    if (e_len) e_len[gw] = e;
-    if (err != HS_OK) report(dev_status, err);
+  // the last warp of (i, b) forms e_len = 1 + sum_{k<K} prod_{j<=k} alpha_j
+  if (__shfl_sync(0xffffffffu, last, 0) && l == 0) {
+    __threadfence();
+    const int64_t ib = r / P;
+    float e = 1.f, prod = 1.f;
+    for (int k = 0; k < P - 1; ++k) {
+      prod *= __ldcg(alpha + ib * P + k);
+      e += prod;
+    }
+    e_len[ib] = e;
   }
+}
+
+// Partials, then one counter per (i, b) at the next 256-byte boundary.
+size_t parts_bytes(int N, int B, int P, int V, int dtype) {
+  const int64_t ch = dtype == HS_FP32 ? chunk_of<HS_FP32>() : chunk_of<HS_BF16>();
+  const int64_t nchunk = (V + ch - 1) / ch;
+  const size_t bytes = size_t(int64_t(B) * P * (int64_t(N) + 1) * nchunk) * sizeof(Part);
+  return (bytes + 255) & ~size_t(255);
 }
 
 template <int DT, bool VEC>
@@ -144,12 +160,17 @@ hs_status launch_t(const void* target, const int32_t* path, int M, const void* d
   Part* parts = static_cast<Part*>(ws);
   const int nchunk = int((V + chunk_of<DT>() - 1) / chunk_of<DT>());
   const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
+  int* counters = e_len ? reinterpret_cast<int*>(static_cast<char*>(ws) +
+                                                  parts_bytes(N, B, P, V, DT))
+                        : nullptr;
   if (launch_pdl(argmax_chunk_kernel<DT, VEC>, dim3(rows, unsigned(nchunk)), dim3(kThreads), 0,
-                 s, target, path, M, drafter, B, P, V, parts, nchunk) != cudaSuccess)
+                 s, target, path, M, drafter, B, P, V, parts, nchunk, counters,
+                 N * B) != cudaSuccess)
     return HS_ERR_CUDA;
-  const int64_t threads = int64_t(N) * B * 32;
+  const int64_t threads = int64_t(N) * B * P * 32;
   if (launch_pdl(greedy_finalize_kernel, dim3(unsigned((threads + 255) / 256)), dim3(256), 0, s,
-                 parts, nchunk, path, M, N, B, P, alpha, e_len, dev_status) != cudaSuccess)
+                 parts, nchunk, path, M, N, B, P, alpha, e_len, counters,
+                 dev_status) != cudaSuccess)
     return HS_ERR_CUDA;
   return HS_OK;
 }
@@ -172,8 +193,7 @@ int64_t chunk_elems(int dtype) {
 }
 
 size_t workspace_bytes(int N, int B, int P, int V, int dtype) {
-  const int64_t nchunk = (V + chunk_elems(dtype) - 1) / chunk_elems(dtype);
-  return size_t(int64_t(B) * P * (int64_t(N) + 1) * nchunk) * sizeof(Part);
+  return parts_bytes(N, B, P, V, dtype) + size_t(N) * B * sizeof(int);
 }
 
 hs_status launch(bool vec, const void* target, const int32_t* path, int M, const void* drafter,
