@@ -929,9 +929,9 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   p.alpha = alpha;
   p.dev_status = dev_status;
   // shapes whose rows the cluster kernel can only spread over part of the
-  // GPU, with enough tiles and rows small enough for L2 to hold every SM's
-  // working set, go to the two-pass kernel on all SMs (measured on
-  // llama3_batch: 344 against 394 us per call)
+  // GPU, with enough drafter rows and rows small enough for L2 to hold every
+  // SM's working set, go to the two-pass kernel on all SMs (measured on
+  // llama3_batch: 317 against 394 us per call)
   int dev = 0, sms = 0, l2 = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
@@ -940,7 +940,7 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   const int cluster_sms =
       pl.C * (dtype == HS_BF16 ? clusters_of<HS_BF16>(pl) : clusters_of<HS_FP16>(pl));
   hs_status st;
-  if (twopass::preferred(V, 2, B * P, sms, cluster_sms, size_t(l2)))
+  if (twopass::preferred(V, 2, B * P, N, sms, cluster_sms, size_t(l2)))
     st = twopass::launch(target, path, M, drafter, dtype, N, B, P, V, c, 0, sms, alpha,
                          dev_status, stream);
   else

@@ -1,22 +1,28 @@
-// hs_twopass.cu -- stochastic feedback (Thm 1), two passes per CTA with the
+// hs_twopass.cu -- stochastic feedback (Thm 1), two passes per row with the
 // second served by L2, for shapes where the cluster kernel (hs_fused.cu)
 // leaves SMs idle and the working set below fits in L2.
 //
-// One CTA per SM, one (b,k) tile at a time, no cluster, no tensor memory;
-// c = log2(e) / T throughout:
-//   A. the target row: offset o_t = c m + log2 sum_v 2^{c z_v - c m}, so that
-//      log2 p_v = c z_v - o_t;
-//   B. per group of up to kG drafters: pass 1 gives each one's offset o_i
-//      the same way; pass 2 walks the rows backwards (the most recently read
-//      part first), reading each target chunk once for the whole group, and
-//      sums  min(p_v, q_v) = 2^{min(c z_t - o_t, c z_d - o_i)}
-//      (2^x is increasing, so the min moves inside: one exp2 per pair).
+// One CTA per SM, no cluster; c = log2(e) / T throughout.
+// The drafter rows of a call, ordered (tile, drafter), are split into even
+// contiguous runs, one per CTA.  A CTA walks its run in groups of up to kG
+// drafters of one tile:
+//   pass 1: the tile's target offset o_t = c m + log2 sum_v 2^{c z_v - c m}
+//           when the group starts a tile (or the run), so that
+//           log2 p_v = c z_v - o_t, then each drafter row's offset o_i;
+//   pass 2: the group's rows walked backwards (the most recently read part
+//           first, while it is still in L2), each target chunk read once
+//           for the group (from tensor memory, see below), summing
+//           min(p_v, q_v) = 2^{min(c z_t - o_t, c z_d - o_i)}
+//           (2^x is increasing, so the min moves inside: one exp2 per pair).
 // One producer warp streams every chunk the consumers need, in their order,
-// into a ring of 32 KB shared-memory stages with cp.async.bulk; the target's
-// loads ask L2 to keep its lines (the row is read 1 + 2 ceil(N/kG) times per
-// tile), pass 2's drafter loads mark theirs as last use.  HBM reads each
-// logit once as long as every SM's target row and kG drafter rows, (1 + kG)
-// rows per SM, stay in L2; the caller checks that (preferred()).
+// into a ring of 32 KB shared-memory stages with cp.async.bulk.  Pass 1 over
+// the target parks its first kTmemChunks chunks (256 KB, a whole 128 256-logit
+// bf16 row) in tensor memory, each thread its own words in its own lane, and
+// pass 2 reads them from there; only the rest of a longer row comes back from
+// L2, its loads asking L2 to keep the lines until the tile's last group.
+// Pass 2's drafter loads mark theirs as last use.  HBM reads each logit once
+// as long as every SM's kG drafter rows and the target's tail stay in L2;
+// the caller checks that (preferred()).
 #include <math.h>
 #include <stdint.h>
 
@@ -34,7 +40,15 @@ constexpr int kStages = 6;                      // ring stages
 constexpr int kVecsPerThread = 4;               // 16-byte vectors of a stage per consumer
 constexpr int kChunkVecs = kVecsPerThread * kConsumers;
 constexpr int kChunkBytes = kChunkVecs * 16;    // 32 KB
-constexpr int kG = 2;                           // drafters per pass-2 group
+constexpr int kG = 2;                           // drafters per group
+constexpr int kWords = 4 * kVecsPerThread;      // 32-bit words of a chunk per thread
+// Tensor memory: 128 lanes x 512 columns of 32 bits.  Consumer warp w owns
+// lanes 32 (w % 4) .. +31 and columns 128 (w / 4) .. +127: kTmemChunks
+// chunks of a row, kWords columns each.
+static_assert(kConsumerWarps % 4 == 0, "warps share the four TMEM lane quadrants evenly");
+constexpr int kTmemColsPerWarp = 512 / (kConsumerWarps / 4);
+constexpr int kTmemChunks = kTmemColsPerWarp / kWords;
+static_assert(kVecsPerThread == 4, "a chunk's words move to tensor memory 16 at a time");
 constexpr long long kTimeoutCycles = 1LL << 31;  // about a second
 
 template <int DT>
@@ -54,18 +68,6 @@ struct Pair<HS_FP16> {
     return __half2float(__ushort_as_half(static_cast<unsigned short>(w >> 16)));
   }
 };
-
-template <int DT>
-__device__ __forceinline__ void unpack(uint4 w, float* x) {
-  x[0] = Pair<DT>::lo(w.x);
-  x[1] = Pair<DT>::hi(w.x);
-  x[2] = Pair<DT>::lo(w.y);
-  x[3] = Pair<DT>::hi(w.y);
-  x[4] = Pair<DT>::lo(w.z);
-  x[5] = Pair<DT>::hi(w.z);
-  x[6] = Pair<DT>::lo(w.w);
-  x[7] = Pair<DT>::hi(w.w);
-}
 
 // ---- PTX wrappers ---------------------------------------------------------------
 
@@ -128,6 +130,39 @@ __device__ __forceinline__ uint4 lds128(uint32_t a) {
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
   return v;
 }
+// ---- tensor memory (the target row between its two passes) ---------------------
+__device__ __forceinline__ void tmem_alloc512(uint32_t dst_smem) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;"
+               :: "r"(dst_smem) : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc512(uint32_t taddr) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" :: "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tmem_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// A chunk's 16 words of this thread into / out of 16 columns of its lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint4 (&v)[4]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, "
+               "%9, %10, %11, %12, %13, %14, %15, %16};"
+               :: "r"(taddr), "r"(v[0].x), "r"(v[0].y), "r"(v[0].z), "r"(v[0].w), "r"(v[1].x),
+                  "r"(v[1].y), "r"(v[1].z), "r"(v[1].w), "r"(v[2].x), "r"(v[2].y), "r"(v[2].z),
+                  "r"(v[2].w), "r"(v[3].x), "r"(v[3].y), "r"(v[3].z), "r"(v[3].w) : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint4 (&v)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, "
+               "%9, %10, %11, %12, %13, %14, %15}, [%16];"
+               : "=r"(v[0].x), "=r"(v[0].y), "=r"(v[0].z), "=r"(v[0].w), "=r"(v[1].x),
+                 "=r"(v[1].y), "=r"(v[1].z), "=r"(v[1].w), "=r"(v[2].x), "=r"(v[2].y),
+                 "=r"(v[2].z), "=r"(v[2].w), "=r"(v[3].x), "=r"(v[3].y), "=r"(v[3].z),
+                 "=r"(v[3].w) : "r"(taddr) : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
 // Barrier of the consumer warps only (the producer warp never joins).
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" :: "n"(kConsumers) : "memory");
@@ -142,12 +177,17 @@ __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2,
   s = a + b;
 }
 
+
+// Per-warp partials of one consumer barrier, double-buffered: buffer b is
+// rewritten two barriers later, after a barrier that every reader of its
+// previous contents has passed.
 struct Shared {
   uint64_t full[kStages], empty[kStages];
-  float m[kConsumerWarps], s[kConsumerWarps];
-  int bad[kConsumerWarps];
-  float acc[kG][kConsumerWarps];
+  float m[2][kConsumerWarps], s[2][kConsumerWarps];
+  int bad[2][kConsumerWarps];
+  float acc[2][kG][kConsumerWarps];
   int error;
+  uint32_t tmem_base;
 };
 
 struct Params {
@@ -160,6 +200,27 @@ struct Params {
   int t0;  // first tile of this kernel; it takes tiles t0 .. B*P-1 (0: all)
   float c;
 };
+
+// A CTA's group: drafters d0 .. d0+dn-1 of one tile, starting at row index
+// r = tile * N + d0 of the run [r, re); up to kG drafters, ending at the
+// tile's last drafter or the run's end.
+// with_t: the group starts a tile or the run, so its pass 1 reads the target.
+struct Group {
+  int tile, d0, dn;
+  bool with_t, t_last;  // t_last: the tile's last group in this run
+};
+__device__ __forceinline__ Group group_at(int r, bool first, int re, int N) {
+  Group g;
+  g.tile = r / N;
+  g.d0 = r - g.tile * N;
+  int dn = kG;
+  if (dn > N - g.d0) dn = N - g.d0;
+  if (dn > re - r) dn = re - r;
+  g.dn = dn;
+  g.with_t = first || g.d0 == 0;
+  g.t_last = g.d0 + dn == N || r + dn == re;
+  return g;
+}
 
 // ---- consumer warps ---------------------------------------------------------------
 
@@ -197,17 +258,108 @@ __device__ __forceinline__ uint32_t pmax(uint32_t a, uint32_t b) {
   return r;
 }
 
-// Per tile, in the producer's order: the target row's offset, then per group
-// each drafter row's offset, then pass 2.  Every consumer thread runs the
-// same control flow (also after a timeout, then on whatever the stages
-// hold), so the consumer barriers always meet; a timed-out call reports
-// HS_ERR_TIMEOUT and writes NaN.  A thread holds 4 vectors (32 logits) of
-// each stage; only a row's last chunk can end early, and only there are the
-// vectors past the row's end replaced by -inf.
+
+// Running statistics of a row in pass 1: the packed running max of the
+// stored words (mw), the scalar max m and offset off = -c m it gives (off
+// stays 0 while the row is all -inf), and the packed partial sums of
+// 2^{c (z - m)}; bad once a NaN or +inf logit was seen.
+struct Stat {
+  uint32_t mw;
+  float m, off;
+  uint64_t s2;
+  bool bad;
+};
+
+template <int DT>
+__device__ __forceinline__ Stat stat_init() {
+  Stat st;
+  st.mw = DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u;
+  st.m = -INFINITY;
+  st.off = 0.f;
+  st.s2 = 0ull;
+  st.bad = false;
+  return st;
+}
+
+// Fold one chunk (the thread's 32 logits) into a row's statistics.  The
+// scalar max is only revisited when the packed max of the words moved.
+template <int DT>
+__device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerThread], float c,
+                                           uint64_t c2) {
+  uint32_t mw = st.mw;
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u)
+    mw = pmax<DT>(mw, pmax<DT>(pmax<DT>(v[u].x, v[u].y), pmax<DT>(v[u].z, v[u].w)));
+  if (mw != st.mw) {
+    st.mw = mw;
+    const float cm = max_nan(Pair<DT>::lo(mw), Pair<DT>::hi(mw));
+    st.bad |= (cm != cm) || cm == INFINITY;
+    if (cm > st.m) {
+      const float r = (st.m == -INFINITY) ? 0.f : ex2((st.m - cm) * c);
+      st.s2 = pack2(lo2(st.s2) * r, hi2(st.s2) * r);
+      st.m = cm;
+      st.off = -cm * c;
+    }
+  }
+  const uint64_t off2 = pack2(st.off, st.off);
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, off2);
+      st.s2 = add2(st.s2, pack2(ex2(lo2(e)), ex2(hi2(e))));
+    }
+  }
+}
+
+// Lane 0 of each warp posts the warp's merged (m, s, bad) of a row.
+__device__ __forceinline__ void post_stat(const Stat& st, float* pm, float* ps, int* pb, int w,
+                                          int l, float c) {
+  float m = st.m, s = lo2(st.s2) + hi2(st.s2);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    merge_ms(m, s, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, s, o), c);
+  const bool bad = __any_sync(0xffffffffu, st.bad);
+  if (l == 0) {
+    pm[w] = m;
+    ps[w] = s;
+    pb[w] = bad;
+  }
+}
+
+// Every thread: the row's offset c M + log2 S from the warps' posts (lanes
+// 0..15 read one each and the warp merges them), NaN for an unusable row.
+__device__ __forceinline__ float row_offset(const float* pm, const float* ps, const int* pb, int l,
+                                            float c) {
+  float m = l < kConsumerWarps ? pm[l] : -INFINITY;
+  float s = l < kConsumerWarps ? ps[l] : 0.f;
+  const bool bad = __any_sync(0xffffffffu, l < kConsumerWarps && pb[l] != 0);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    merge_ms(m, s, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, s, o), c);
+  if (bad || m == -INFINITY || !(s > 0.f) || isinf(s)) return __int_as_float(0x7fc00000);
+  return fmaf(m, c, __log2f(s));
+}
+
+// The consumers' side of drafter rows rb .. re-1, group by group in the
+// producer's order: pass 1 over the target row (when the group starts a
+// tile or the run; its first kTmemChunks chunks also go to tensor memory)
+// and over each drafter row, then pass 2 backwards, each target chunk (from
+// tensor memory, or the ring past kTmemChunks) followed by the group's
+// drafter chunks.  Every consumer
+// thread runs the same control flow (also after a timeout, then on whatever
+// the stages hold), so the consumer barriers always meet; a timed-out call
+// reports HS_ERR_TIMEOUT and writes NaN.  A thread holds 4 vectors (32
+// logits) of each stage; only a row's last chunk can end early, and only
+// there are the vectors past the row's end replaced by -inf.
 template <int DT>
 __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t ring0, int nvec,
-                                         int nch, int T, float c, volatile int* err) {
+                                         int nch, int rb, int re, float c, volatile int* err) {
   const int t = threadIdx.x, w = t >> 5, l = t & 31;
+  const uint32_t tcol = sh.tmem_base + (uint32_t(32 * (w & 3)) << 16) +
+                        uint32_t(kTmemColsPerWarp * (w >> 2));  // this thread's lane and columns
+  const int T = p.B * p.P;
   uint32_t stage = 0, phase = 0;  // the next stage and its phase parity
   bool ok = true;
   const uint32_t ninf = DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u;
@@ -229,124 +381,107 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       phase ^= 1u;
     }
   };
-  // a whole row: offset c m + log2 sum 2^{c (z - m)}, NaN for an unusable row
-  auto row_offset = [&]() -> float {
-    float m = -INFINITY;
-    uint64_t s2 = 0ull;  // packed partial sums relative to m
-    bool bad = false;
+  uint32_t rp = 0;  // partial buffer of the next consumer barrier
+  // pass 1 over one row: its offset in every thread, NaN for an unusable row;
+  // park: the row's first kTmemChunks chunks also go to tensor memory
+  auto pass1 = [&](bool park) -> float {
+    Stat st = stat_init<DT>();
     for (int ch = 0; ch < nch; ++ch) {
       uint4 v[kVecsPerThread];
       take(ch, v);
-      uint32_t mw = pmax<DT>(pmax<DT>(v[0].x, v[0].y), pmax<DT>(v[0].z, v[0].w));
+      if (park && ch < kTmemChunks) tmem_st16(tcol + uint32_t(kWords * ch), v);
+      stat_chunk<DT>(st, v, c, c2);
+    }
+    if (park) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    post_stat(st, sh.m[rp], sh.s[rp], sh.bad[rp], w, l, c);
+    consumer_sync();
+    const float o = row_offset(sh.m[rp], sh.s[rp], sh.bad[rp], l, c);
+    rp ^= 1u;
+    return o;
+  };
+  float ot = 0.f;         // offset of the current tile's target row
+  bool bad_path = false;  // the current tile has an out-of-range path node
+  bool first = true;
+  for (int r = rb; r < re;) {
+    const Group g = group_at(r, first, re, p.N);
+    if (g.with_t) {
+      bad_path = false;
+      (void)target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path);
+      ot = pass1(true);
+    }
+    float od[kG];
 #pragma unroll
-      for (int u = 1; u < kVecsPerThread; ++u)
-        mw = pmax<DT>(mw, pmax<DT>(pmax<DT>(v[u].x, v[u].y), pmax<DT>(v[u].z, v[u].w)));
-      const float cm = max_nan(Pair<DT>::lo(mw), Pair<DT>::hi(mw));
-      bad |= (cm != cm) || cm == INFINITY;
-      if (cm > m) {
-        const float r = (m == -INFINITY) ? 0.f : ex2((m - cm) * c);
-        s2 = pack2(lo2(s2) * r, hi2(s2) * r);
-        m = cm;
-      }
-      if (m != -INFINITY) {
-        const float off = -m * c;
-        const uint64_t off2 = pack2(off, off);
+    for (int gi = 0; gi < kG; ++gi) od[gi] = gi < g.dn ? pass1(false) : 0.f;
+    uint64_t acc[kG];
 #pragma unroll
-        for (int u = 0; u < kVecsPerThread; ++u) {
-          const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+    for (int gi = 0; gi < kG; ++gi) acc[gi] = 0ull;
+    const uint64_t ot2 = pack2(-ot, -ot);
+    for (int ch = nch - 1; ch >= 0; --ch) {
+      uint4 v[kVecsPerThread];
+      if (ch < kTmemChunks)
+        tmem_ld16(tcol + uint32_t(kWords * ch), v);
+      else
+        take(ch, v);
+      float xt[8 * kVecsPerThread];  // log2 p of the thread's 32 logits
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, off2);
-            s2 = add2(s2, pack2(ex2(lo2(e)), ex2(hi2(e))));
-          }
+      for (int u = 0; u < kVecsPerThread; ++u) {
+        const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, ot2);
+          xt[8 * u + 2 * q] = lo2(e);
+          xt[8 * u + 2 * q + 1] = hi2(e);
         }
       }
-    }
-    float s = lo2(s2) + hi2(s2);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-      merge_ms(m, s, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, s, o), c);
-    bad = __any_sync(0xffffffffu, bad);
-    if (l == 0) {
-      sh.m[w] = m;
-      sh.s[w] = s;
-      sh.bad[w] = bad;
-    }
-    consumer_sync();
-    float M = sh.m[0], S = sh.s[0];
-    bool B = sh.bad[0];
-    for (int q = 1; q < kConsumerWarps; ++q) {
-      merge_ms(M, S, sh.m[q], sh.s[q], c);
-      B = B || sh.bad[q];
-    }
-    consumer_sync();  // the partials are reused by the next reduction
-    if (B || M == -INFINITY || !(S > 0.f) || isinf(S)) return __int_as_float(0x7fc00000);
-    return fmaf(M, c, __log2f(S));
-  };
-  for (int tile = p.t0 + blockIdx.x; tile < T; tile += gridDim.x) {
-    bool bad_path = false;
-    (void)target_row<DT>(p.target, p.path, p.M, p.P, tile, p.V, &bad_path);
-    const float ot = row_offset();
-    const uint64_t ot2 = pack2(-ot, -ot);
-    for (int g0 = 0; g0 < p.N; g0 += kG) {
-      const int gn = p.N - g0 < kG ? p.N - g0 : kG;
-      float od[kG];
-      uint64_t acc[kG];
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
-        od[gi] = gi < gn ? row_offset() : 0.f;
-        acc[gi] = 0ull;
-      }
-      for (int ch = nch - 1; ch >= 0; --ch) {
-        uint4 v[kVecsPerThread];
-        take(ch, v);
-        float xt[8 * kVecsPerThread];  // log2 p of the thread's 32 logits
+        if (gi < g.dn) {
+          take(ch, v);
+          const uint64_t od2 = pack2(-od[gi], -od[gi]);
 #pragma unroll
-        for (int u = 0; u < kVecsPerThread; ++u) {
-          const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+          for (int u = 0; u < kVecsPerThread; ++u) {
+            const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, ot2);
-            xt[8 * u + 2 * q] = lo2(e);
-            xt[8 * u + 2 * q + 1] = hi2(e);
-          }
-        }
-#pragma unroll
-        for (int gi = 0; gi < kG; ++gi) {
-          if (gi < gn) {
-            take(ch, v);
-            const uint64_t od2 = pack2(-od[gi], -od[gi]);
-#pragma unroll
-            for (int u = 0; u < kVecsPerThread; ++u) {
-              const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2);
-                acc[gi] = add2(acc[gi], pack2(ex2(fminf(xt[8 * u + 2 * q], lo2(e))),
-                                              ex2(fminf(xt[8 * u + 2 * q + 1], hi2(e)))));
-              }
+            for (int q = 0; q < 4; ++q) {
+              const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2);
+              acc[gi] = add2(acc[gi], pack2(ex2(fminf(xt[8 * u + 2 * q], lo2(e))),
+                                            ex2(fminf(xt[8 * u + 2 * q + 1], hi2(e)))));
             }
           }
         }
       }
+    }
+#pragma unroll
+    for (int gi = 0; gi < kG; ++gi) {
+      if (gi < g.dn) {
+        const float a = warp_sum(lo2(acc[gi]) + hi2(acc[gi]));
+        if (l == 0) sh.acc[rp][gi][w] = a;
+      }
+    }
+    consumer_sync();
+    if (w == 0) {
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
-        const float a = warp_sum(lo2(acc[gi]) + hi2(acc[gi]));
-        if (l == 0) sh.acc[gi][w] = a;
-      }
-      consumer_sync();
-      if (t == 0) {
-        for (int gi = 0; gi < gn; ++gi) {
-          float a = 0.f;
-          for (int q = 0; q < kConsumerWarps; ++q) a += sh.acc[gi][q];
-          const bool good = ok && !bad_path && !(ot != ot) && !(od[gi] != od[gi]);
-          if (!good && ok) report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
-          p.alpha[int64_t(g0 + gi) * T + tile] = good ? a : __int_as_float(0x7fc00000);
+        if (gi < g.dn) {
+          const float a = warp_sum(l < kConsumerWarps ? sh.acc[rp][gi][l] : 0.f);
+          if (l == 0) {
+            const bool fine = ok && *err == 0;
+            const bool good = fine && !bad_path && !(ot != ot) && !(od[gi] != od[gi]);
+            if (!good && fine) report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
+            p.alpha[int64_t(g.d0 + gi) * T + g.tile] = good ? a : __int_as_float(0x7fc00000);
+          }
         }
       }
-      consumer_sync();
     }
+    rp ^= 1u;
+    r += g.dn;
+    first = false;
   }
+  // every consumer warp is done with tensor memory before it is released
+  tmem_fence_before();
+  consumer_sync();
+  tmem_fence_after();
+  if (w == 0) tmem_dealloc512(sh.tmem_base);
 }
 
 size_t shared_bytes() {
@@ -367,28 +502,36 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
     sh.error = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  // The shared memory keeps this kernel to one CTA per SM, so the allocation
+  // can only wait for another kernel's CTA on the SM to finish.
+  if (warp == 0) tmem_alloc512(saddr(&sh.tmem_base));
+  tmem_fence_before();
   __syncthreads();
+  tmem_fence_after();
   pdl_wait();  // the set-up above overlaps the previous kernel of the stream
   volatile int* err = &sh.error;
   const int nvec = p.V / 8;
   const int nch = (nvec + kChunkVecs - 1) / kChunkVecs;
   const int T = p.B * p.P;
+  // this CTA's run of drafter rows (tile-major): an even split of rows
+  // t0*N .. T*N-1
+  const int64_t first = int64_t(p.t0) * p.N, total = int64_t(T - p.t0) * p.N;
+  const int rb = int(first + total * blockIdx.x / gridDim.x);
+  const int re = int(first + total * (blockIdx.x + 1) / gridDim.x);
   const float c = p.c;
 
   if (warp == kConsumerWarps) {
     // ------------------------------ producer ---------------------------------
-    // Streams every chunk in the order the consumers take them: the target
-    // row; then per group, each drafter row; then the rows backwards, each
-    // target chunk followed by the group's drafter chunks.
+    // Streams every chunk in the order the consumers take them (see consumer).
     if (lane == 0) {
       const uint64_t normal = make_policy(0), keep = make_policy(1), once = make_policy(2);
-      uint32_t k = 0;
+      uint32_t n = 0;  // chunks issued
       bool ok = true;
       auto put = [&](const char* row, int ch, uint64_t pol) {
         if (!ok) return;
-        const uint32_t s = k % kStages;
-        if (k >= kStages &&
-            !mbar_wait(saddr(&sh.empty[s]), ((k / kStages) - 1) & 1u, err, p.dev_status)) {
+        const uint32_t s = n % kStages;
+        if (n >= kStages &&
+            !mbar_wait(saddr(&sh.empty[s]), ((n / kStages) - 1) & 1u, err, p.dev_status)) {
           ok = false;
           return;
         }
@@ -396,31 +539,33 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
         const int nv = nvec - v0 < kChunkVecs ? nvec - v0 : kChunkVecs;
         bulk_fill(ring0 + s * kChunkBytes, saddr(&sh.full[s]), row + int64_t(v0) * 16,
                   uint32_t(nv) * 16u, pol);
-        ++k;
+        ++n;
       };
-      for (int tile = p.t0 + blockIdx.x; tile < T; tile += gridDim.x) {
+      auto drow = [&](int d, int tile) {
+        return static_cast<const char*>(row_ptr<DT>(p.drafter, int64_t(d) * T + tile, p.V));
+      };
+      bool first_group = true;
+      for (int r = rb; r < re;) {
+        const Group g = group_at(r, first_group, re, p.N);
         bool bad_path = false;
-        const char* trow = static_cast<const char*>(
-            target_row<DT>(p.target, p.path, p.M, p.P, tile, p.V, &bad_path));
-        for (int ch = 0; ch < nch; ++ch) put(trow, ch, keep);
-        for (int g0 = 0; g0 < p.N; g0 += kG) {
-          const int gn = p.N - g0 < kG ? p.N - g0 : kG;
-          for (int gi = 0; gi < gn; ++gi) {
-            const char* drow = static_cast<const char*>(
-                row_ptr<DT>(p.drafter, int64_t(g0 + gi) * T + tile, p.V));
-            for (int ch = 0; ch < nch; ++ch) put(drow, ch, normal);
-          }
-          for (int ch = nch - 1; ch >= 0; --ch) {
-            put(trow, ch, keep);
-            for (int gi = 0; gi < gn; ++gi)
-              put(static_cast<const char*>(row_ptr<DT>(p.drafter, int64_t(g0 + gi) * T + tile, p.V)),
-                  ch, once);
-          }
+        const char* tr = static_cast<const char*>(
+            target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path));
+        if (g.with_t)  // chunks past kTmemChunks are read again in pass 2
+          for (int ch = 0; ch < nch; ++ch) put(tr, ch, ch < kTmemChunks ? once : keep);
+        for (int gi = 0; gi < g.dn; ++gi) {
+          const char* dr = drow(g.d0 + gi, g.tile);
+          for (int ch = 0; ch < nch; ++ch) put(dr, ch, normal);
         }
+        for (int ch = nch - 1; ch >= 0; --ch) {
+          if (ch >= kTmemChunks) put(tr, ch, g.t_last ? once : keep);
+          for (int gi = 0; gi < g.dn; ++gi) put(drow(g.d0 + gi, g.tile), ch, once);
+        }
+        r += g.dn;
+        first_group = false;
       }
       if (!ok) {
         // the copies already issued must land before the CTA's memory goes
-        for (uint32_t j = k > uint32_t(kStages) ? k - kStages : 0; j < k; ++j) {
+        for (uint32_t j = n > uint32_t(kStages) ? n - kStages : 0; j < n; ++j) {
           const long long t0 = clock64();
           while (!mbar_test(saddr(&sh.full[j % kStages]), (j / kStages) & 1u) &&
                  clock64() - t0 < kTimeoutCycles) {
@@ -429,15 +574,19 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
       }
     }
   } else {
-    consumer<DT>(p, sh, ring0, nvec, nch, T, c, err);
+    consumer<DT>(p, sh, ring0, nvec, nch, rb, re, c, err);
   }
 }
 
 }  // namespace
 
-bool preferred(int V, int elem_bytes, int tiles, int sms, int cluster_sms, size_t l2_bytes) {
-  if (cluster_sms >= sms || tiles < 2 * sms) return false;
-  const double working_set = double(1 + kG) * double(V) * elem_bytes * sms;
+bool preferred(int V, int elem_bytes, int tiles, int N, int sms, int cluster_sms,
+               size_t l2_bytes) {
+  if (cluster_sms >= sms || int64_t(tiles) * N < 2 * int64_t(sms)) return false;
+  // per SM: kG drafter rows and the part of the target row past tensor memory
+  const double row = double(V) * elem_bytes;
+  const double tail = row - double(kTmemChunks) * kChunkBytes;
+  const double working_set = (kG * row + (tail > 0 ? tail : 0.0)) * sms;
   return working_set <= 0.9 * double(l2_bytes);
 }
 
@@ -469,3 +618,4 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
 
 }  // namespace twopass
 }  // namespace hs
+

@@ -12,12 +12,16 @@ namespace hs {
 namespace twopass {
 
 // Whether this kernel should take a call: the cluster kernel would leave
-// SMs idle (cluster_sms < sms), every SM gets at least two tiles, and the
-// rows each SM keeps in L2 between its two passes fit in 90% of L2.
-bool preferred(int V, int elem_bytes, int tiles, int sms, int cluster_sms, size_t l2_bytes);
+// SMs idle (cluster_sms < sms), there are at least two drafter rows per SM,
+// and what each SM keeps in L2 between a row's two passes -- two drafter
+// rows and the part of the target row tensor memory does not hold (all past
+// 256 KB) -- fits in 90% of L2.
+bool preferred(int V, int elem_bytes, int tiles, int N, int sms, int cluster_sms,
+               size_t l2_bytes);
 
-// alpha of tiles t0 .. B*P-1 (bf16/fp16, V % 8 == 0, 16-byte-aligned rows),
-// one CTA per tile at a time over `grid` CTAs (one per SM).
+// alpha of tiles t0 .. B*P-1 (bf16/fp16, V % 8 == 0, 16-byte-aligned rows)
+// over `grid` CTAs (one per SM), each taking an even, contiguous run of the
+// drafter rows (tile-major).
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
                  int N, int B, int P, int V, float c, int t0, int grid, float* alpha,
                  int* dev_status, cudaStream_t stream);

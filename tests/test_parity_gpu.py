@@ -317,3 +317,25 @@ def test_two_pass_kernel_flags_bad_rows():
     a, e, st = run(t, 1.0, False)
     assert st == hf.HS_ERR_INVALID_ARG
     assert np.isnan(a[:, 79, 2]).all() and np.isnan(a).sum() == 2
+
+
+def test_two_pass_kernel_groups_cross_tiles():
+    """N = 5 drafters: the 1600 drafter rows are split evenly over the SMs in
+    runs that start and end inside tiles (such a run reads the tile's target
+    row again), walked in groups of two, of one at a tile's end and at the
+    start of an odd CTA's run; every alpha and e_len is compared."""
+    w = synth.Workload("two_pass", N=5, B=64, P=5, V=76808, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=44)
+    compare_full(d, 0.9, False)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp16"])
+def test_two_pass_kernel_qwen_vocab(dtype):
+    """Qwen-vocabulary rows (V = 151936) and 960 drafter rows: the target row
+    is longer than the 256 KB tensor memory holds, so pass 2 reads its first
+    eight chunks from tensor memory and the last two from the ring."""
+    w = synth.Workload("two_pass", N=3, B=40, P=8, V=151936, dtype=dtype, temperature=0.7,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=45)
+    compare_full(d, 0.7, False)
