@@ -133,22 +133,24 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
                :: "r"(bar), "r"(bytes) : "memory");
 }
-// try_wait suspends the thread until the phase completes or about 1 ms has
-// passed, so a waiting warp does not spin through the issue slots.
+// try_wait suspends the thread until the phase completes or a system-chosen
+// time limit passes, so a waiting warp does not spin through the issue slots.
+// (Without a time-limit operand: on the two-pass kernel that form measured
+// fewer instructions and 3% less time than a 1 ms limit.)
 __device__ __forceinline__ bool mbar_test_cta(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile("{\n\t.reg .pred p;\n\t"
-               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
                "selp.u32 %0, 1, 0, p;\n\t}"
-               : "=r"(ok) : "r"(bar), "r"(parity), "r"(1000000u) : "memory");
+               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
   return ok != 0;
 }
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile("{\n\t.reg .pred p;\n\t"
-               "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+               "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
                "selp.u32 %0, 1, 0, p;\n\t}"
-               : "=r"(ok) : "r"(bar), "r"(parity), "r"(1000000u) : "memory");
+               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
   return ok != 0;
 }
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,

@@ -83,9 +83,9 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile("{\n\t.reg .pred p;\n\t"
-               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
                "selp.u32 %0, 1, 0, p;\n\t}"
-               : "=r"(ok) : "r"(bar), "r"(parity), "r"(1000000u) : "memory");
+               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
   return ok != 0;
 }
 // Bounded wait; false (the CTA's error flag set, a timeout reported) after
@@ -167,16 +167,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint4 (&v)[4]) {
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" :: "n"(kConsumers) : "memory");
 }
-
-// Merge running pairs (m, s): s is relative to m, in 2^{c(.)}.
-__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c) {
-  const float M = max_nan(m, m2);
-  const float a = (m == -INFINITY) ? 0.f : s * ex2((m - M) * c);
-  const float b = (m2 == -INFINITY) ? 0.f : s2 * ex2((m2 - M) * c);
-  m = M;
-  s = a + b;
-}
-
 
 // Per-warp partials of one consumer barrier, double-buffered: buffer b is
 // rewritten two barriers later, after a barrier that every reader of its
@@ -313,13 +303,24 @@ __device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerTh
   }
 }
 
+// Every lane: the merge (M, S) of the warp's pairs (m, s), each s relative
+// to its m in 2^{c(.)}: the max first, then every sum rescaled to it once and
+// added up.  (m is never NaN; a +inf m only comes with the row's bad flag.)
+__device__ __forceinline__ void warp_merge(float& m, float& s, float c) {
+  float M = m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  s = (m == -INFINITY) ? 0.f : s * ex2((m - M) * c);
+  m = M;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+}
+
 // Lane 0 of each warp posts the warp's merged (m, s, bad) of a row.
 __device__ __forceinline__ void post_stat(const Stat& st, float* pm, float* ps, int* pb, int w,
                                           int l, float c) {
   float m = st.m, s = lo2(st.s2) + hi2(st.s2);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-    merge_ms(m, s, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, s, o), c);
+  warp_merge(m, s, c);
   const bool bad = __any_sync(0xffffffffu, st.bad);
   if (l == 0) {
     pm[w] = m;
@@ -335,9 +336,7 @@ __device__ __forceinline__ float row_offset(const float* pm, const float* ps, co
   float m = l < kConsumerWarps ? pm[l] : -INFINITY;
   float s = l < kConsumerWarps ? ps[l] : 0.f;
   const bool bad = __any_sync(0xffffffffu, l < kConsumerWarps && pb[l] != 0);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-    merge_ms(m, s, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, s, o), c);
+  warp_merge(m, s, c);
   if (bad || m == -INFINITY || !(s > 0.f) || isinf(s)) return __int_as_float(0x7fc00000);
   return fmaf(m, c, __log2f(s));
 }
@@ -364,12 +363,14 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
   bool ok = true;
   const uint32_t ninf = DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u;
   const uint64_t c2 = pack2(c, c);
-  auto take = [&](int ch, uint4 (&v)[kVecsPerThread]) {
+  // the next stage into v; tail: the row's last chunk, whose vectors past
+  // the row's end become -inf (callers pass a constant, ch == nch - 1)
+  auto take = [&](int ch, bool tail, uint4 (&v)[kVecsPerThread]) {
     if (!mbar_wait(saddr(&sh.full[stage]), phase, err, p.dev_status)) ok = false;
     const uint32_t base = ring0 + stage * kChunkBytes + uint32_t(t) * 16u;
 #pragma unroll
     for (int u = 0; u < kVecsPerThread; ++u) v[u] = lds128(base + uint32_t(u * kConsumers) * 16u);
-    if (ch == nch - 1) {
+    if (tail) {
 #pragma unroll
       for (int u = 0; u < kVecsPerThread; ++u)
         if (ch * kChunkVecs + u * kConsumers + t >= nvec) v[u] = make_uint4(ninf, ninf, ninf, ninf);
@@ -386,12 +387,14 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
   // park: the row's first kTmemChunks chunks also go to tensor memory
   auto pass1 = [&](bool park) -> float {
     Stat st = stat_init<DT>();
-    for (int ch = 0; ch < nch; ++ch) {
+    auto step = [&](int ch, bool tail) {
       uint4 v[kVecsPerThread];
-      take(ch, v);
+      take(ch, tail, v);
       if (park && ch < kTmemChunks) tmem_st16(tcol + uint32_t(kWords * ch), v);
       stat_chunk<DT>(st, v, c, c2);
-    }
+    };
+    for (int ch = 0; ch < nch - 1; ++ch) step(ch, false);
+    step(nch - 1, true);
     if (park) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
     post_stat(st, sh.m[rp], sh.s[rp], sh.bad[rp], w, l, c);
     consumer_sync();
@@ -416,12 +419,15 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) acc[gi] = 0ull;
     const uint64_t ot2 = pack2(-ot, -ot);
-    for (int ch = nch - 1; ch >= 0; --ch) {
+    // one chunk of pass 2: the target's words from tensor memory (tm) or the
+    // ring, then each drafter's from the ring (callers pass constant tail and
+    // tm where they can, so the loops below carry neither test)
+    auto p2chunk = [&](int ch, bool tail, bool tm) {
       uint4 v[kVecsPerThread];
-      if (ch < kTmemChunks)
+      if (tm)
         tmem_ld16(tcol + uint32_t(kWords * ch), v);
       else
-        take(ch, v);
+        take(ch, tail, v);
       float xt[8 * kVecsPerThread];  // log2 p of the thread's 32 logits
 #pragma unroll
       for (int u = 0; u < kVecsPerThread; ++u) {
@@ -436,7 +442,7 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
         if (gi < g.dn) {
-          take(ch, v);
+          take(ch, tail, v);
           const uint64_t od2 = pack2(-od[gi], -od[gi]);
 #pragma unroll
           for (int u = 0; u < kVecsPerThread; ++u) {
@@ -450,7 +456,11 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
           }
         }
       }
-    }
+    };
+    p2chunk(nch - 1, true, nch - 1 < kTmemChunks);
+    int ch = nch - 2;
+    for (; ch >= kTmemChunks; --ch) p2chunk(ch, false, false);
+    for (; ch >= 0; --ch) p2chunk(ch, false, true);
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) {
       if (gi < g.dn) {
