@@ -249,63 +249,89 @@ __device__ __forceinline__ uint32_t pmax(uint32_t a, uint32_t b) {
 }
 
 
-// Running statistics of a row in pass 1: the packed running max of the
-// stored words (mw), the scalar max m and offset off = -c m it gives (off
-// stays 0 while the row is all -inf), and the packed partial sums of
-// 2^{c (z - m)}; bad once a NaN or +inf logit was seen.
+// Running statistics of a row in pass 1: a reference m taken from the row's
+// own logits (-inf until one is seen), off = -c m (0 before that), and two
+// independent chains of packed partial sums of 2^{c z - off}; bad once a NaN
+// or +inf logit was seen.  Any reference from the data gives the same offset
+// c m + log2 sum_v 2^{c (z_v - m)}; it only has to keep the terms finite,
+// so it is the max of the first chunk and grows only when a chunk's sum
+// passes 2^100 (a term above 2^126 would overflow).  Terms far below it
+// vanish as they would below the row max, which is at least as large.
 struct Stat {
-  uint32_t mw;
   float m, off;
-  uint64_t s2;
+  uint64_t s2[2];
   bool bad;
 };
 
 template <int DT>
 __device__ __forceinline__ Stat stat_init() {
   Stat st;
-  st.mw = DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u;
   st.m = -INFINITY;
   st.off = 0.f;
-  st.s2 = 0ull;
+  st.s2[0] = st.s2[1] = 0ull;
   st.bad = false;
   return st;
 }
 
-// Fold one chunk (the thread's 32 logits) into a row's statistics.  The
-// scalar max is only revisited when the packed max of the words moved.
+// The chunk's (the thread's 32 logits) sums of 2^{c z - off}, two packed pairs.
 template <int DT>
-__device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerThread], float c,
-                                           uint64_t c2) {
-  uint32_t mw = st.mw;
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u)
-    mw = pmax<DT>(mw, pmax<DT>(pmax<DT>(v[u].x, v[u].y), pmax<DT>(v[u].z, v[u].w)));
-  if (mw != st.mw) {
-    st.mw = mw;
-    const float cm = max_nan(Pair<DT>::lo(mw), Pair<DT>::hi(mw));
-    st.bad |= (cm != cm) || cm == INFINITY;
-    if (cm > st.m) {
-      const float r = (st.m == -INFINITY) ? 0.f : ex2((st.m - cm) * c);
-      st.s2 = pack2(lo2(st.s2) * r, hi2(st.s2) * r);
-      st.m = cm;
-      st.off = -cm * c;
-    }
-  }
-  const uint64_t off2 = pack2(st.off, st.off);
+__device__ __forceinline__ void chunk_sums(const uint4 (&v)[kVecsPerThread], uint64_t c2,
+                                           float off, uint64_t& a, uint64_t& b) {
+  const uint64_t off2 = pack2(off, off);
+  a = b = 0ull;
 #pragma unroll
   for (int u = 0; u < kVecsPerThread; ++u) {
     const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, off2);
-      st.s2 = add2(st.s2, pack2(ex2(lo2(e)), ex2(hi2(e))));
+      const uint64_t x = pack2(ex2(lo2(e)), ex2(hi2(e)));
+      if (q & 1)
+        b = add2(b, x);
+      else
+        a = add2(a, x);
     }
   }
 }
 
+// Fold one chunk into a row's statistics.  The chunk's max is only formed
+// for the first chunk with a finite logit and when the sums under the
+// current reference pass 2^100 or are not finite (NaN / +inf logits).
+template <int DT>
+__device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerThread], float c,
+                                           uint64_t c2) {
+  uint64_t a, b;
+  bool redo = st.m == -INFINITY;
+  if (!redo) {
+    chunk_sums<DT>(v, c2, st.off, a, b);
+    const uint64_t t2 = add2(a, b);
+    redo = !(lo2(t2) + hi2(t2) <= 0x1p100f);
+  }
+  if (redo) {
+    uint32_t mw = pmax<DT>(pmax<DT>(v[0].x, v[0].y), pmax<DT>(v[0].z, v[0].w));
+#pragma unroll
+    for (int u = 1; u < kVecsPerThread; ++u)
+      mw = pmax<DT>(mw, pmax<DT>(pmax<DT>(v[u].x, v[u].y), pmax<DT>(v[u].z, v[u].w)));
+    const float cm = max_nan(Pair<DT>::lo(mw), Pair<DT>::hi(mw));
+    st.bad |= (cm != cm) || cm == INFINITY;
+    if (cm > st.m) {
+      const float r = (st.m == -INFINITY) ? 0.f : ex2((st.m - cm) * c);
+      const uint64_t r2 = pack2(r, r), z2 = 0ull;
+      st.s2[0] = fma2(st.s2[0], r2, z2);
+      st.s2[1] = fma2(st.s2[1], r2, z2);
+      st.m = cm;
+      st.off = -cm * c;
+    }
+    chunk_sums<DT>(v, c2, st.off, a, b);
+  }
+  st.s2[0] = add2(st.s2[0], a);
+  st.s2[1] = add2(st.s2[1], b);
+}
+
 // Every lane: the merge (M, S) of the warp's pairs (m, s), each s relative
-// to its m in 2^{c(.)}: the max first, then every sum rescaled to it once and
-// added up.  (m is never NaN; a +inf m only comes with the row's bad flag.)
+// to its reference m in 2^{c(.)}: the largest reference first, then every sum
+// rescaled to it once and added up.  (m is never NaN; a +inf m only comes
+// with the row's bad flag.)
 __device__ __forceinline__ void warp_merge(float& m, float& s, float c) {
   float M = m;
 #pragma unroll
@@ -319,7 +345,8 @@ __device__ __forceinline__ void warp_merge(float& m, float& s, float c) {
 // Lane 0 of each warp posts the warp's merged (m, s, bad) of a row.
 __device__ __forceinline__ void post_stat(const Stat& st, float* pm, float* ps, int* pb, int w,
                                           int l, float c) {
-  float m = st.m, s = lo2(st.s2) + hi2(st.s2);
+  const uint64_t s2 = add2(st.s2[0], st.s2[1]);
+  float m = st.m, s = lo2(s2) + hi2(s2);
   warp_merge(m, s, c);
   const bool bad = __any_sync(0xffffffffu, st.bad);
   if (l == 0) {
@@ -415,14 +442,15 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     float od[kG];
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) od[gi] = gi < g.dn ? pass1(false) : 0.f;
-    uint64_t acc[kG];
+    uint64_t acc[kG][2];  // two independent chains per drafter
 #pragma unroll
-    for (int gi = 0; gi < kG; ++gi) acc[gi] = 0ull;
+    for (int gi = 0; gi < kG; ++gi) acc[gi][0] = acc[gi][1] = 0ull;
     const uint64_t ot2 = pack2(-ot, -ot);
     // one chunk of pass 2: the target's words from tensor memory (tm) or the
-    // ring, then each drafter's from the ring (callers pass constant tail and
-    // tm where they can, so the loops below carry neither test)
-    auto p2chunk = [&](int ch, bool tail, bool tm) {
+    // ring, then each drafter's from the ring; full: the group has kG
+    // drafters (callers pass constants where they can, so the loops below
+    // carry none of these tests)
+    auto p2chunk = [&](int ch, bool tail, bool tm, bool full) {
       uint4 v[kVecsPerThread];
       if (tm)
         tmem_ld16(tcol + uint32_t(kWords * ch), v);
@@ -441,7 +469,7 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       }
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
-        if (gi < g.dn) {
+        if (full || gi < g.dn) {
           take(ch, tail, v);
           const uint64_t od2 = pack2(-od[gi], -od[gi]);
 #pragma unroll
@@ -450,21 +478,28 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2);
-              acc[gi] = add2(acc[gi], pack2(ex2(fminf(xt[8 * u + 2 * q], lo2(e))),
+              acc[gi][q & 1] = add2(acc[gi][q & 1], pack2(ex2(fminf(xt[8 * u + 2 * q], lo2(e))),
                                             ex2(fminf(xt[8 * u + 2 * q + 1], hi2(e)))));
             }
           }
         }
       }
     };
-    p2chunk(nch - 1, true, nch - 1 < kTmemChunks);
-    int ch = nch - 2;
-    for (; ch >= kTmemChunks; --ch) p2chunk(ch, false, false);
-    for (; ch >= 0; --ch) p2chunk(ch, false, true);
+    auto pass2 = [&](bool full) {
+      p2chunk(nch - 1, true, nch - 1 < kTmemChunks, full);
+      int ch = nch - 2;
+      for (; ch >= kTmemChunks; --ch) p2chunk(ch, false, false, full);
+      for (; ch >= 0; --ch) p2chunk(ch, false, true, full);
+    };
+    if (g.dn == kG)
+      pass2(true);
+    else
+      pass2(false);
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) {
       if (gi < g.dn) {
-        const float a = warp_sum(lo2(acc[gi]) + hi2(acc[gi]));
+        const uint64_t a2 = add2(acc[gi][0], acc[gi][1]);
+        const float a = warp_sum(lo2(a2) + hi2(a2));
         if (l == 0) sh.acc[rp][gi][w] = a;
       }
     }

@@ -306,11 +306,13 @@ def test_two_pass_kernel_flags_bad_rows():
     w = synth.Workload("two_pass", N=2, B=80, P=4, V=76808, dtype="bf16", temperature=1.0,
                        target="zipf", sigma="qwen")
     d = synth.make_inputs(w, device=DEV, seed=42)
-    d["drafter"][1, 77, 3, 5] = float("nan")
+    d["drafter"][1, 77, 3, 5] = float("nan")      # in a row's first chunk
+    d["drafter"][0, 12, 1, 70000] = float("inf")  # in a late chunk
     a, e, st = run(d, 1.0, False)
     ra, re, rst = oracle_feedback(d, 1.0, False)
     assert st == hf.HS_ERR_NONFINITE
-    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 1
+    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 2
+    assert np.isnan(a[1, 77, 3]) and np.isnan(a[0, 12, 1])
     assert_rel(a, ra, RTOL_ALPHA, "alpha next to a NaN row")
     t = synth.make_inputs(W["tree_path"], device=DEV, B=80, N=2, V=76808, seed=43)
     t["path"][79, 2] = 999
@@ -339,3 +341,19 @@ def test_two_pass_kernel_qwen_vocab(dtype):
                        target="zipf", sigma="qwen")
     d = synth.make_inputs(w, device=DEV, seed=45)
     compare_full(d, 0.7, False)
+
+
+@pytest.mark.parametrize("T", [0.05, 5.0])
+def test_two_pass_kernel_row_extremes(T):
+    """The two-pass kernel at extreme temperatures on rows whose largest
+    logits sit at the end of the vocabulary (so the first chunk's max is a
+    low reference that later chunks must raise), with the first 40000 logits
+    of one query's rows masked to -inf; every alpha and e_len is compared."""
+    w = synth.Workload("two_pass", N=2, B=80, P=4, V=76808, dtype="bf16", temperature=T,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=46)
+    d["target"] = torch.flip(d["target"], dims=[-1]).contiguous()
+    d["drafter"] = torch.flip(d["drafter"], dims=[-1]).contiguous()
+    d["target"][3, :, :40000] = float("-inf")
+    d["drafter"][:, 3, :, :40000] = float("-inf")
+    compare_full(d, T, False)
