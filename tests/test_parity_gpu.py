@@ -230,9 +230,11 @@ def test_full_size_greedy_everything():
 
 # ---- both feedback paths ------------------------------------------------------
 # bf16/fp16 rows with V % 8 == 0, 16-byte-aligned logits and N <= 32 take the
-# single-read cluster kernel (cluster size 1, 2, 4 or 8 by V) up to
-# V = 153600 and the persistent streaming kernel above; everything else takes
-# the two-pass kernels.  These cases cross each boundary.
+# single-read cluster kernel (the cluster size, up to 16, that keeps the most
+# SMs busy) up to V = 153600 -- or the two-pass-per-SM kernel when there are at
+# least two drafter rows per SM and its L2 working set fits -- and the
+# persistent streaming kernel above; everything else takes the fallback
+# two-pass kernels.  These cases cross each boundary.
 
 @pytest.mark.parametrize("V", [8, 4096, 19200, 19208, 38400, 38408, 76800, 76808, 128256,
                                151936, 153600, 153608, 262144])
