@@ -359,3 +359,14 @@ def test_two_pass_kernel_row_extremes(T):
     d["target"][3, :, :40000] = float("-inf")
     d["drafter"][:, 3, :, :40000] = float("-inf")
     compare_full(d, T, False)
+
+
+@pytest.mark.parametrize("V", [38408, 65536])
+def test_two_pass_kernel_short_rows(V):
+    """The shortest rows the two-pass kernel takes (the cluster kernel needs 3
+    or 4 CTAs per row there, leaving SMs idle): three chunks with a ragged
+    tail (V = 38408), and four full chunks (V = 65536)."""
+    w = synth.Workload("two_pass", N=3, B=64, P=5, V=V, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=47 + V)
+    compare_full(d, 0.9, False)
