@@ -50,6 +50,7 @@ constexpr int kTmemColsPerWarp = 512 / (kConsumerWarps / 4);
 constexpr int kTmemChunks = kTmemColsPerWarp / kWords;
 static_assert(kVecsPerThread == 4, "a chunk's words move to tensor memory 16 at a time");
 constexpr long long kTimeoutCycles = 1LL << 31;  // about a second
+constexpr float kFoldLimit = 64.f;  // |o| below which pass 2 folds R + L into one offset
 
 template <int DT>
 struct Pair;  // two logits of a 32-bit word as floats
@@ -249,16 +250,18 @@ __device__ __forceinline__ uint32_t pmax(uint32_t a, uint32_t b) {
 }
 
 
-// Running statistics of a row in pass 1: a reference m taken from the row's
-// own logits (-inf until one is seen), off = -c m (0 before that), and two
-// independent chains of packed partial sums of 2^{c z - off}; bad once a NaN
-// or +inf logit was seen.  Any reference from the data gives the same offset
-// c m + log2 sum_v 2^{c (z_v - m)}; it only has to keep the terms finite,
-// so it is the max of the first chunk and grows only when a chunk's sum
-// passes 2^100 (a term above 2^126 would overflow).  Terms far below it
-// vanish as they would below the row max, which is at least as large.
+// Running statistics of a row in pass 1, in log2 units: an integer reference
+// R (-inf until the row shows a finite logit) and two independent chains of
+// packed partial sums of 2^{c z - R}; bad once a NaN or +inf logit was seen.
+// R = ceil(c m) for m the max of the chunk that set it, so every offset and
+// every rescale between references is exact and the sums are exactly
+// relative to R (up to the rounding of each term).  Any reference gives the
+// same normaliser R + log2 sum_v 2^{c z_v - R}; R only has to keep the terms
+// finite, so it is set by the first chunk with a finite logit and raised only
+// when a chunk's sum under it passes 2^100 (a term above 2^126 would
+// overflow).  Terms far below R vanish as they would below the row max.
 struct Stat {
-  float m, off;
+  float R;
   uint64_t s2[2];
   bool bad;
 };
@@ -266,17 +269,17 @@ struct Stat {
 template <int DT>
 __device__ __forceinline__ Stat stat_init() {
   Stat st;
-  st.m = -INFINITY;
-  st.off = 0.f;
+  st.R = -INFINITY;
   st.s2[0] = st.s2[1] = 0ull;
   st.bad = false;
   return st;
 }
 
-// The chunk's (the thread's 32 logits) sums of 2^{c z - off}, two packed pairs.
+// The chunk's (the thread's 32 logits) sums of 2^{c z - R}, two packed pairs.
 template <int DT>
 __device__ __forceinline__ void chunk_sums(const uint4 (&v)[kVecsPerThread], uint64_t c2,
-                                           float off, uint64_t& a, uint64_t& b) {
+                                           float R, uint64_t& a, uint64_t& b) {
+  const float off = R == -INFINITY ? 0.f : -R;  // all -inf so far: every term is 0
   const uint64_t off2 = pack2(off, off);
   a = b = 0ull;
 #pragma unroll
@@ -301,9 +304,9 @@ template <int DT>
 __device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerThread], float c,
                                            uint64_t c2) {
   uint64_t a, b;
-  bool redo = st.m == -INFINITY;
+  bool redo = st.R == -INFINITY;
   if (!redo) {
-    chunk_sums<DT>(v, c2, st.off, a, b);
+    chunk_sums<DT>(v, c2, st.R, a, b);
     const uint64_t t2 = add2(a, b);
     redo = !(lo2(t2) + hi2(t2) <= 0x1p100f);
   }
@@ -314,58 +317,67 @@ __device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerTh
       mw = pmax<DT>(mw, pmax<DT>(pmax<DT>(v[u].x, v[u].y), pmax<DT>(v[u].z, v[u].w)));
     const float cm = max_nan(Pair<DT>::lo(mw), Pair<DT>::hi(mw));
     st.bad |= (cm != cm) || cm == INFINITY;
-    if (cm > st.m) {
-      const float r = (st.m == -INFINITY) ? 0.f : ex2((st.m - cm) * c);
+    const float Rn = ceilf(cm * c);  // -inf for an all -inf chunk, NaN stays out below
+    if (Rn > st.R) {
+      const float r = (st.R == -INFINITY) ? 0.f : ex2(st.R - Rn);  // an exact power of 2
       const uint64_t r2 = pack2(r, r), z2 = 0ull;
       st.s2[0] = fma2(st.s2[0], r2, z2);
       st.s2[1] = fma2(st.s2[1], r2, z2);
-      st.m = cm;
-      st.off = -cm * c;
+      st.R = Rn;
     }
-    chunk_sums<DT>(v, c2, st.off, a, b);
+    chunk_sums<DT>(v, c2, st.R, a, b);
   }
   st.s2[0] = add2(st.s2[0], a);
   st.s2[1] = add2(st.s2[1], b);
 }
 
-// Every lane: the merge (M, S) of the warp's pairs (m, s), each s relative
-// to its reference m in 2^{c(.)}: the largest reference first, then every sum
-// rescaled to it once and added up.  (m is never NaN; a +inf m only comes
-// with the row's bad flag.)
-__device__ __forceinline__ void warp_merge(float& m, float& s, float c) {
-  float M = m;
+// Every lane: the merge (R, S) of the warp's pairs (R, s), each s relative to
+// its integer reference R: the largest reference first, then every sum
+// rescaled to it once (by an exact power of 2) and added up.  (R is never
+// NaN; a +inf R only comes with the row's bad flag.)
+__device__ __forceinline__ void warp_merge(float& R, float& s) {
+  float M = R;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  s = (m == -INFINITY) ? 0.f : s * ex2((m - M) * c);
-  m = M;
+  s = (R == -INFINITY) ? 0.f : s * ex2(R - M);
+  R = M;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
 }
 
-// Lane 0 of each warp posts the warp's merged (m, s, bad) of a row.
+// Lane 0 of each warp posts the warp's merged (R, s, bad) of a row.
 __device__ __forceinline__ void post_stat(const Stat& st, float* pm, float* ps, int* pb, int w,
-                                          int l, float c) {
+                                          int l) {
   const uint64_t s2 = add2(st.s2[0], st.s2[1]);
-  float m = st.m, s = lo2(s2) + hi2(s2);
-  warp_merge(m, s, c);
+  float R = st.R, s = lo2(s2) + hi2(s2);
+  warp_merge(R, s);
   const bool bad = __any_sync(0xffffffffu, st.bad);
   if (l == 0) {
-    pm[w] = m;
+    pm[w] = R;
     ps[w] = s;
     pb[w] = bad;
   }
 }
 
-// Every thread: the row's offset c M + log2 S from the warps' posts (lanes
-// 0..15 read one each and the warp merges them), NaN for an unusable row.
-__device__ __forceinline__ float row_offset(const float* pm, const float* ps, const int* pb, int l,
-                                            float c) {
-  float m = l < kConsumerWarps ? pm[l] : -INFINITY;
+// A row's normaliser in log2 units, as its integer reference R and
+// L = log2 sum_v 2^{c z_v - R}: log2 p_v = c z_v - R - L.  Both NaN for an
+// unusable row (a NaN or +inf logit, or no finite logit).
+struct Norm {
+  float R, L;
+};
+
+// Every thread: the row's Norm from the warps' posts (lanes 0..15 read one
+// each and the warp merges them).
+__device__ __forceinline__ Norm row_norm(const float* pm, const float* ps, const int* pb, int l) {
+  float R = l < kConsumerWarps ? pm[l] : -INFINITY;
   float s = l < kConsumerWarps ? ps[l] : 0.f;
   const bool bad = __any_sync(0xffffffffu, l < kConsumerWarps && pb[l] != 0);
-  warp_merge(m, s, c);
-  if (bad || m == -INFINITY || !(s > 0.f) || isinf(s)) return __int_as_float(0x7fc00000);
-  return fmaf(m, c, __log2f(s));
+  warp_merge(R, s);
+  if (bad || R == -INFINITY || !(s > 0.f) || isinf(s)) {
+    const float nan = __int_as_float(0x7fc00000);
+    return Norm{nan, nan};
+  }
+  return Norm{R, __log2f(s)};
 }
 
 // The consumers' side of drafter rows rb .. re-1, group by group in the
@@ -410,9 +422,9 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     }
   };
   uint32_t rp = 0;  // partial buffer of the next consumer barrier
-  // pass 1 over one row: its offset in every thread, NaN for an unusable row;
-  // park: the row's first kTmemChunks chunks also go to tensor memory
-  auto pass1 = [&](bool park) -> float {
+  // pass 1 over one row: its normaliser in every thread (NaN for an unusable
+  // row); park: the row's first kTmemChunks chunks also go to tensor memory
+  auto pass1 = [&](bool park) -> Norm {
     Stat st = stat_init<DT>();
     auto step = [&](int ch, bool tail) {
       uint4 v[kVecsPerThread];
@@ -423,13 +435,13 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     for (int ch = 0; ch < nch - 1; ++ch) step(ch, false);
     step(nch - 1, true);
     if (park) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-    post_stat(st, sh.m[rp], sh.s[rp], sh.bad[rp], w, l, c);
+    post_stat(st, sh.m[rp], sh.s[rp], sh.bad[rp], w, l);
     consumer_sync();
-    const float o = row_offset(sh.m[rp], sh.s[rp], sh.bad[rp], l, c);
+    const Norm n = row_norm(sh.m[rp], sh.s[rp], sh.bad[rp], l);
     rp ^= 1u;
-    return o;
+    return n;
   };
-  float ot = 0.f;         // offset of the current tile's target row
+  Norm nt = {0.f, 0.f};   // normaliser of the current tile's target row
   bool bad_path = false;  // the current tile has an out-of-range path node
   bool first = true;
   for (int r = rb; r < re;) {
@@ -437,20 +449,40 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     if (g.with_t) {
       bad_path = false;
       (void)target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path);
-      ot = pass1(true);
+      nt = pass1(true);
     }
-    float od[kG];
+    Norm nd[kG];
 #pragma unroll
-    for (int gi = 0; gi < kG; ++gi) od[gi] = gi < g.dn ? pass1(false) : 0.f;
+    for (int gi = 0; gi < kG; ++gi) nd[gi] = gi < g.dn ? pass1(false) : Norm{0.f, 0.f};
+    // The folded form takes each row's normaliser as one offset o = R + L,
+    // held in fp32 to ulp(o)/2: alpha stays within 2.6e-6 relative while
+    // |o| < kFoldLimit.  Otherwise (low temperatures, large logits) pass 2
+    // keeps R and L apart: the target's terms use R_t alone, each drafter's
+    // are shifted by L_t - L_d (a small number, full precision), and alpha
+    // is scaled by 2^{-L_t} at the end.  NaN normalisers take the split form
+    // and are flagged below.
+    bool split = !(fabsf(nt.R + nt.L) < kFoldLimit);
+#pragma unroll
+    for (int gi = 0; gi < kG; ++gi)
+      if (gi < g.dn) split |= !(fabsf(nd[gi].R + nd[gi].L) < kFoldLimit);
+    const float tofs = split ? nt.R : nt.R + nt.L;
+    const uint64_t ot2 = pack2(-tofs, -tofs);
+    uint64_t od2[kG], sh2[kG];
+#pragma unroll
+    for (int gi = 0; gi < kG; ++gi) {
+      const float dofs = split ? nd[gi].R : nd[gi].R + nd[gi].L;
+      const float shift = split ? nt.L - nd[gi].L : 0.f;
+      od2[gi] = pack2(-dofs, -dofs);
+      sh2[gi] = pack2(shift, shift);
+    }
     uint64_t acc[kG][2];  // two independent chains per drafter
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) acc[gi][0] = acc[gi][1] = 0ull;
-    const uint64_t ot2 = pack2(-ot, -ot);
     // one chunk of pass 2: the target's words from tensor memory (tm) or the
     // ring, then each drafter's from the ring; full: the group has kG
-    // drafters (callers pass constants where they can, so the loops below
-    // carry none of these tests)
-    auto p2chunk = [&](int ch, bool tail, bool tm, bool full) {
+    // drafters; sp: the split form (callers pass constants where they can, so
+    // the loops below carry none of these tests)
+    auto p2chunk = [&](int ch, bool tail, bool tm, bool full, bool sp) {
       uint4 v[kVecsPerThread];
       if (tm)
         tmem_ld16(tcol + uint32_t(kWords * ch), v);
@@ -471,13 +503,13 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       for (int gi = 0; gi < kG; ++gi) {
         if (full || gi < g.dn) {
           take(ch, tail, v);
-          const uint64_t od2 = pack2(-od[gi], -od[gi]);
 #pragma unroll
           for (int u = 0; u < kVecsPerThread; ++u) {
             const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-              const uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2);
+              uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2[gi]);
+              if (sp) e = add2(e, sh2[gi]);
               acc[gi][q & 1] = add2(acc[gi][q & 1], pack2(ex2(fminf(xt[8 * u + 2 * q], lo2(e))),
                                             ex2(fminf(xt[8 * u + 2 * q + 1], hi2(e)))));
             }
@@ -485,16 +517,16 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
         }
       }
     };
-    auto pass2 = [&](bool full) {
-      p2chunk(nch - 1, true, nch - 1 < kTmemChunks, full);
+    auto pass2 = [&](bool full, bool sp) {
+      p2chunk(nch - 1, true, nch - 1 < kTmemChunks, full, sp);
       int ch = nch - 2;
-      for (; ch >= kTmemChunks; --ch) p2chunk(ch, false, false, full);
-      for (; ch >= 0; --ch) p2chunk(ch, false, true, full);
+      for (; ch >= kTmemChunks; --ch) p2chunk(ch, false, false, full, sp);
+      for (; ch >= 0; --ch) p2chunk(ch, false, true, full, sp);
     };
-    if (g.dn == kG)
-      pass2(true);
+    if (!split)
+      pass2(g.dn == kG, false);  // the usual case: one drafter pair form per group
     else
-      pass2(false);
+      pass2(g.dn == kG, true);
 #pragma unroll
     for (int gi = 0; gi < kG; ++gi) {
       if (gi < g.dn) {
@@ -508,10 +540,11 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
         if (gi < g.dn) {
-          const float a = warp_sum(l < kConsumerWarps ? sh.acc[rp][gi][l] : 0.f);
+          float a = warp_sum(l < kConsumerWarps ? sh.acc[rp][gi][l] : 0.f);
+          if (split) a *= ex2(-nt.L);
           if (l == 0) {
             const bool fine = ok && *err == 0;
-            const bool good = fine && !bad_path && !(ot != ot) && !(od[gi] != od[gi]);
+            const bool good = fine && !bad_path && !(nt.L != nt.L) && !(nd[gi].L != nd[gi].L);
             if (!good && fine) report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
             p.alpha[int64_t(g.d0 + gi) * T + g.tile] = good ? a : __int_as_float(0x7fc00000);
           }

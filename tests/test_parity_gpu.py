@@ -370,3 +370,26 @@ def test_two_pass_kernel_short_rows(V):
                        target="zipf", sigma="qwen")
     d = synth.make_inputs(w, device=DEV, seed=47 + V)
     compare_full(d, 0.9, False)
+
+
+@pytest.mark.parametrize("T", [0.05, 0.5])
+def test_two_pass_kernel_large_logits(T):
+    """Logits three times the synthetic scale (max around 30): at these
+    temperatures a row's log2 normaliser reaches the hundreds, where one fp32
+    offset would hold it only to ~3e-5; the kernel keeps its integer reference
+    and log2-sum apart there, and every alpha stays within 1e-5 relative.
+    Some pairs are nearly disjoint (alpha ~1e-41): terms below the fp32 normal
+    range, 2^-126, flush to zero (ex2.approx.ftz), so the comparison also
+    allows V * 2^-126 ~ 1e-33 absolute."""
+    w = synth.Workload("two_pass", N=2, B=80, P=4, V=76808, dtype="bf16", temperature=T,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=48)
+    d["target"] = (d["target"].float() * 3).to(torch.bfloat16)
+    d["drafter"] = (d["drafter"].float() * 3).to(torch.bfloat16)
+    a, e, st = run(d, T, False)
+    ra, re, rst = oracle_feedback(d, T, False)
+    assert st == hf.HS_OK and rst == 0
+    floor = w.V * 2.0 ** -126
+    assert_rel(a, ra, RTOL_ALPHA, "alpha", atol=floor)
+    assert_rel(e, re, RTOL_ALPHA, "e_len")
+    assert np.nanmax(ra) > 0.1, "some pairs must overlap well above the flush floor"
