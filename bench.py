@@ -45,7 +45,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = ("drafter-position-vocab evals/s and achieved HBM GB/s (% of GB300 peak) "
           "per hs_feedback")
-DEFAULT_WORKLOAD = "qwen3_8b_chain"
+DEFAULT_WORKLOAD = "long_session"
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -62,6 +62,11 @@ def parse_args():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--clock-preload-s", type=float, default=1.5,
+                    help="seconds of untimed step replays before the timed region, under "
+                         "the clock sampler")
+    ap.add_argument("--cpu-budget-s", type=float, default=8.0,
+                    help="seconds of oracle work per CPU-baseline leg (1 thread, all cores)")
     ap.add_argument("--session", action="store_true",
                     help="long-session learner run: cumulative regret over the workload's rounds")
     ap.add_argument("--rounds", type=int, default=0, help="session rounds (0: the workload's)")
@@ -197,34 +202,91 @@ def oracle_alpha(o, w, args):
     return lambda t, d: o.alpha_pair(t, d, w.temperature, greedy)
 
 
-def oracle_sample(w, sets, args, budget_s=10.0):
-    """The fp64 C oracle (single-threaded, as it stands) on whole (b,k)
-    tiles of the first input set until ~budget_s seconds of CPU work."""
-    import oracle
+def host_cpu() -> dict:
+    """The host's usable core count and CPU model (lscpu), recorded beside
+    the oracle's timings."""
+    try:
+        cores = len(os.sched_getaffinity(0))
+    except AttributeError:
+        cores = os.cpu_count() or 1
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return {"nproc": cores, "model": model, "machine": os.uname().machine}
+
+
+def oracle_tiles(w, d):
+    """(target row, drafter rows) of every (b,k) tile of one input set, as
+    the stored bytes the oracle reads."""
     from paper_2510_20064_gb300 import synth
-    o = oracle.get()
-    pair = oracle_alpha(o, w, args)
-    d = sets[0]
     t_all = synth.storage_numpy(d["target"])
     path = d.get("path")
     path_np = None if path is None else path.cpu().numpy()
-    evals, tiles, t_used = 0, 0, 0.0
-    tile = 0
-    while t_used < budget_s:
-        b, k = divmod(tile % (w.B * w.P), w.P)
+    B = d["drafter"].shape[1]
+    for tile in range(B * w.P):
+        b, k = divmod(tile, w.P)
         trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
-        drows = synth.storage_numpy(d["drafter"][:, b, k])
-        t0 = time.perf_counter()
-        for i in range(w.N):
-            pair(trow, drows[i])
-        t_used += time.perf_counter() - t0
-        evals += w.N * w.V
-        tiles += 1
-        tile += 1
-    return {"value": evals / t_used, "unit": "evals/s", "cores": 1, "kind": "oracle",
-            "sample": f"{tiles} (b,k) tiles (cycling over the {w.B * w.P} of one input set) x "
-                      f"{w.N} drafters x V={w.V} of the {w.name} workload, fp64 C oracle, "
-                      f"1 thread, {t_used:.1f} s"}
+        yield trow, synth.storage_numpy(d["drafter"][:, b, k])
+
+
+def oracle_rate(w, tiles, args, threads: int, budget_s: float):
+    """The fp64 C oracle as it stands, on whole (b,k) tiles cycled from
+    `tiles`, on `threads` host threads for about budget_s seconds: each
+    thread takes one drafter row at a time (rows in parallel, each row's sums
+    sequential inside the oracle; ctypes releases the GIL during the call).
+    Returns (evals/s, rows done, seconds)."""
+    import concurrent.futures as cf
+    import threading
+
+    import oracle
+    o = oracle.get()
+    pair = oracle_alpha(o, w, args)
+    rows = [(t, dr[i]) for t, dr in tiles for i in range(w.N)]
+    lock = threading.Lock()
+    counter = [0]
+    t_start = time.perf_counter()
+    deadline = t_start + budget_s
+
+    def worker():
+        done = 0
+        while time.perf_counter() < deadline:
+            with lock:
+                j = counter[0]
+                counter[0] += 1
+            t, d = rows[j % len(rows)]
+            pair(t, d)
+            done += 1
+        return done
+
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        done = sum(ex.map(lambda _: worker(), range(threads)))
+    elapsed = time.perf_counter() - t_start
+    return done * w.V / elapsed, done, elapsed
+
+
+def oracle_sample(w, sets, args):
+    """The fp64 C oracle (as it stands) on whole (b,k) tiles of the first
+    input set: once on 1 thread and once on every host core, each for
+    --cpu-budget-s seconds."""
+    host = host_cpu()
+    tiles = []
+    for tile in oracle_tiles(w, sets[0]):
+        tiles.append(tile)
+        if len(tiles) >= 4 * host["nproc"]:  # enough distinct rows to keep every core busy
+            break
+    v1, n1, s1 = oracle_rate(w, tiles, args, 1, args.cpu_budget_s)
+    vall, nall, sall = oracle_rate(w, tiles, args, host["nproc"], args.cpu_budget_s)
+    return {"value": vall, "unit": "evals/s", "cores": host["nproc"], "kind": "oracle",
+            "value_1_core": v1, "host": host,
+            "sample": f"{nall} drafter rows (all cores) and {n1} rows (1 core) cycling over "
+                      f"{len(tiles)} (b,k) tiles x {w.N} drafters x V={w.V} of the {w.name} "
+                      f"workload, fp64 C oracle, {sall:.1f} s / {s1:.1f} s"}
 
 
 # ---- the benchmark -------------------------------------------------------------
@@ -325,14 +387,30 @@ def run_ours(args):
                 fn(sets[s % n_sets])
         return g
 
-    def timed(fn, steps):
+    def timed(fn, steps, preload_s=0.0):
         full, rem = divmod(steps, per_graph)
         g_full = capture(fn, per_graph) if full else None
         g_rem = capture(fn, rem) if rem else None
+        g_any = g_full or g_rem
         with torch.cuda.stream(stream):
             for _ in range(2):  # graph warm-up
-                (g_full or g_rem).replay()
+                g_any.replay()
         stream.synchronize()
+        if preload_s > 0:
+            # keep the GPU busy for preload_s right before the timed region,
+            # so that the clock samples describe the kernels under load
+            w0 = torch.cuda.Event(enable_timing=True)
+            w1 = torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                w0.record(stream)
+                g_any.replay()
+                w1.record(stream)
+            stream.synchronize()
+            per_replay = max(w0.elapsed_time(w1) / 1e3, 1e-6)
+            with torch.cuda.stream(stream):
+                for _ in range(int(math.ceil(preload_s / per_replay))):
+                    g_any.replay()
+            stream.synchronize()
         hdist.barrier(world, dev)
         torch.cuda.synchronize(dev)
         t0 = torch.cuda.Event(enable_timing=True)
@@ -350,8 +428,11 @@ def run_ours(args):
 
     clocks = ClockSampler(gpu_uuid(dev))
     clocks.start()
-    t_step = timed(step, args.steps)
+    t_step = timed(step, args.steps, preload_s=args.clock_preload_s)
     clk = clocks.stop()
+    if clk is not None:
+        clk["window"] = (f"{args.clock_preload_s:.1f} s of step-graph replays right before the "
+                         "timed region, then the timed region")
     t_fb = timed(feedback, args.steps)
     t_learn = timed(token_learner, args.steps) if token else None
     assert int(status.item()) == 0, hf.hs_status_string(int(status.item()))
@@ -436,40 +517,45 @@ def run_ours(args):
 
 
 def run_reference(args):
-    """The fp64 CPU oracle on the host cores, same metric and config."""
+    """The fp64 CPU oracle on every host core, same metric and config: each
+    step is a bounded sample of the workload, enough whole (b,k) tiles for
+    one drafter row per core, the rows run in parallel (ctypes releases the
+    GIL during each oracle call)."""
     from paper_2510_20064_gb300 import dist as hdist
     rank, world, _ = hdist.rank_info()
     if rank != 0:
         return
+    import concurrent.futures as cf
+
     import oracle
-    import torch
     from paper_2510_20064_gb300 import synth
     w = synth.WORKLOADS[args.workload]
-    d = synth.make_inputs(w, device="cpu", B=min(w.B, 2))
+    host = host_cpu()
+    cores = host["nproc"]
+    tiles_per_step = max(1, math.ceil(cores / w.N))
+    d = synth.make_inputs(w, device="cpu", B=min(w.B, max(2, math.ceil(2 * tiles_per_step / w.P))))
+    tiles = list(oracle_tiles(w, d))
     o = oracle.get()
     pair = oracle_alpha(o, w, args)
-    t_all = synth.storage_numpy(d["target"])
-    path = d.get("path")
-    path_np = None if path is None else path.numpy()
-    tiles = [(b, k) for b in range(d["drafter"].shape[1]) for k in range(w.P)]
 
-    def one(s):
-        b, k = tiles[s % len(tiles)]
-        trow = t_all[b, path_np[b, k]] if path_np is not None else t_all[b, k]
-        drows = synth.storage_numpy(d["drafter"][:, b, k])
-        for i in range(w.N):
-            pair(trow, drows[i])
+    def one(ex, s):
+        rows = []
+        for j in range(tiles_per_step):
+            t, dr = tiles[(s * tiles_per_step + j) % len(tiles)]
+            rows.extend((t, dr[i]) for i in range(w.N))
+        list(ex.map(lambda td: pair(*td), rows))
 
-    for s in range(args.warmup):
-        one(s)
-    t0 = time.perf_counter()
-    for s in range(args.steps):
-        one(s)
-    t = time.perf_counter() - t0
-    value = args.steps * w.N * w.V / t
-    sample = (f"each step = one (b,k) tile of {w.name}: {w.N} drafter rows x V={w.V}, "
-              "fp64 C oracle, 1 thread")
-    del torch
+    with cf.ThreadPoolExecutor(max_workers=cores) as ex:
+        for s in range(args.warmup):
+            one(ex, s)
+        t0 = time.perf_counter()
+        for s in range(args.steps):
+            one(ex, args.warmup + s)
+        t = time.perf_counter() - t0
+    evals_step = tiles_per_step * w.N * w.V
+    value = args.steps * evals_step / t
+    sample = (f"each step = {tiles_per_step} (b,k) tile(s) of {w.name}: {tiles_per_step * w.N} "
+              f"drafter rows x V={w.V}, fp64 C oracle, rows in parallel on {cores} threads")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "evals/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -477,8 +563,8 @@ def run_reference(args):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "N": w.N, "B": w.B, "K": w.K, "V": w.V,
                    "mode": args.mode, "branch_l": args.branch_l if args.mode == "topl" else None},
-        "cpu_baseline": {"value": value, "unit": "evals/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "evals/s", "cores": cores, "kind": "oracle",
+                         "sample": sample, "host": host},
         "e2e": {"value": value, "unit": "evals/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)

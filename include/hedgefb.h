@@ -123,7 +123,11 @@ hs_status hs_feedback(const void* target, const void* drafter, int dtype, int N,
  *    return HS_ERR_UNSUPPORTED before any launch.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress, with that device current); make that first call
- *    before capturing a stream into a CUDA graph.
+ *    before capturing a stream into a CUDA graph.  The address belongs to
+ *    the device's current context: every call compares that context's id
+ *    with the one the address was found in, and a device reset (which
+ *    replaces the context) makes the next call look it up again, so that
+ *    call, too, belongs before any capture.
  *  - Every call on a device shares the one array, which keeps the last
  *    call's contents; whatever must start at zero is cleared by the call
  *    itself.  Calls whose executions overlap on the GPU (different streams,

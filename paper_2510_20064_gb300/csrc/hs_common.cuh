@@ -10,6 +10,7 @@
 namespace hs {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kMaxDevices = 64;  // devices a host-side launch cache keeps entries for
 
 // ---- programmatic dependent launch ------------------------------------------
 // Every kernel here is launched with programmatic stream serialization, so

@@ -31,6 +31,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "hs_common.cuh"
 #include "hs_fused.h"
 #include "hs_twopass.h"
@@ -797,33 +799,44 @@ void fill_config(cudaLaunchConfig_t& cfg, cudaLaunchAttribute (&attr)[2], const 
 }
 
 // Resident clusters of fused_kernel<DT, U> with clusters of pl.C CTAs (0 when
-// none fit).  Each cluster size is queried once, on the first call, so that
-// later calls can be captured into CUDA graphs; the kernel's attributes
-// (shared memory, non-portable cluster sizes) are raised once as well.
+// none fit) on the current device.  Each (device, cluster size) is queried
+// once, on its first call, so that later calls can be captured into CUDA
+// graphs; the kernel's attributes (shared memory, non-portable cluster
+// sizes) are raised once per device as well.  The cache is keyed by device
+// and guarded by a mutex, so host threads driving different GPUs may call
+// concurrently.
 template <int DT, int U>
 int resident_clusters(const Plan& pl) {
   auto kern = fused_kernel<DT, U>;
   const size_t smem = shared_bytes(U);
-  static bool configured = false;
-  if (!configured) {
+  struct Cache {
+    bool configured;
+    int resident[kMaxRanks + 1];  // 0: not queried yet, -1: none fit
+  };
+  static std::mutex mu;
+  static Cache cache[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  Cache& c = cache[dev];
+  if (!c.configured) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) !=
             cudaSuccess ||
         cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
             cudaSuccess)
       return 0;
-    configured = true;
+    c.configured = true;
   }
-  static int resident[kMaxRanks + 1] = {};  // 0: not queried yet, -1: none fit
-  if (resident[pl.C] == 0) {
+  if (c.resident[pl.C] == 0) {
     cudaLaunchConfig_t cfg;
     cudaLaunchAttribute attr[2];
     fill_config<DT, U>(cfg, attr, pl, smem, nullptr);
     int n = 0;
-    resident[pl.C] = (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0)
-                         ? n
-                         : -1;
+    c.resident[pl.C] = (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0)
+                           ? n
+                           : -1;
   }
-  return resident[pl.C] > 0 ? resident[pl.C] : 0;
+  return c.resident[pl.C] > 0 ? c.resident[pl.C] : 0;
 }
 
 template <int DT>

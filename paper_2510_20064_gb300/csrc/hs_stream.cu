@@ -23,6 +23,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "hs_common.cuh"
 #include "hs_stream.h"
 
@@ -335,14 +337,26 @@ Layout layout(int N, int B, int P, int V) {
 template <int DT>
 hs_status launch_t(const Params& p0, void* ws, cudaStream_t stream) {
   auto kern = stream_kernel<DT>;
-  static int per_sm = 0, nsm = 0;  // occupancy: queried on the first call
-  if (!per_sm) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0) != cudaSuccess ||
-        per_sm < 1)
-      return HS_ERR_CUDA;
+  // occupancy and SM count, queried on the first call per device (so that
+  // later calls can be captured into CUDA graphs); the mutex lets host
+  // threads driving different GPUs call concurrently
+  static std::mutex mu;
+  static int per_sm_of[kMaxDevices] = {}, nsm_of[kMaxDevices] = {};
+  int dev = 0, per_sm = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return HS_ERR_CUDA;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (!per_sm_of[dev]) {
+      int ps = 0, n = 0;
+      if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+          cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, kern, kThreads, 0) != cudaSuccess ||
+          ps < 1)
+        return HS_ERR_CUDA;
+      per_sm_of[dev] = ps;
+      nsm_of[dev] = n;
+    }
+    per_sm = per_sm_of[dev];
+    nsm = nsm_of[dev];
   }
   Params p = p0;
   // one step of items must stay in L2 until its overlap: bound the grid so

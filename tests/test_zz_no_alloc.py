@@ -18,7 +18,7 @@ import torch
 
 import paper_2510_20064_gb300 as hf
 from paper_2510_20064_gb300 import synth
-from parity_util import RTOL_ALPHA, assert_rel, to_np
+from parity_util import to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -60,8 +60,10 @@ def test_static_matches_hs_feedback(name, sizes, greedy):
         torch.cuda.synchronize()
         assert st == hf.HS_OK, hf.hs_status_string(st)
         assert int(status.item()) == hf.HS_OK
-        assert_rel(to_np(alpha), ref_a[-1], RTOL_ALPHA, f"{name} alpha, call {call}")
-        assert_rel(to_np(e_len), ref_e[-1], RTOL_ALPHA, f"{name} e_len, call {call}")
+        # the same kernels on the same bytes: results are identical, so any
+        # leftover of the previous call in the shared scratch would show
+        assert np.array_equal(to_np(alpha), ref_a[-1], equal_nan=True), f"{name} alpha, call {call}"
+        assert np.array_equal(to_np(e_len), ref_e[-1], equal_nan=True), f"{name} e_len, call {call}"
     assert not np.array_equal(ref_a[0], ref_a[1]), "the two calls must see different inputs"
 
 
