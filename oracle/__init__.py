@@ -52,6 +52,8 @@ def _bind(lib):
         "orc_topl_set": ([P, I, I, I, P], None),
         "orc_alpha_topl": ([P, P, I, I, D, I, I, P], I),
         "orc_feedback_topl": ([P, P, I, P, I, I, I, I, I, D, I, I, P, P], I),
+        "orc_alpha_topl_pruned": ([P, P, I, I, D, I, I, I, P], I),
+        "orc_feedback_topl_pruned": ([P, P, I, P, I, I, I, I, I, D, I, I, P, P, P], I),
         "orc_hedge": ([P, I, D, P, P], None),
         "orc_normalhedge": ([P, P, P, I, P, P], I),
         "orc_learner_step": ([P, P, I, I, I, I, I, D, P, P, P, P, P], I),
@@ -219,6 +221,42 @@ class Oracle:
         st = self.lib.orc_feedback_topl(_ptr(target), None if pp is None else _ptr(pp), M,
                                         _ptr(drafter), dtype_code(target), N, B, P, V, float(T),
                                         int(bool(greedy)), int(L), _ptr(alpha), _ptr(e_len))
+        return alpha, e_len, st
+
+    def alpha_topl_pruned(self, zt: np.ndarray, zd: np.ndarray, T: float, greedy: bool, L: int,
+                          keep: int):
+        zt = np.ascontiguousarray(zt)
+        zd = np.ascontiguousarray(zd)
+        a = ctypes.c_double()
+        st = self.lib.orc_alpha_topl_pruned(_ptr(zt), _ptr(zd), dtype_code(zt), zt.shape[-1],
+                                            float(T), int(bool(greedy)), int(L), int(keep),
+                                            ctypes.byref(a))
+        return a.value, st
+
+    def feedback_topl_pruned(self, target: np.ndarray, drafter: np.ndarray, T: float,
+                             greedy: bool, L: int, keep: np.ndarray,
+                             path: np.ndarray | None = None):
+        """feedback_topl() with the dynamically pruned candidate sets: the
+        first keep[i,b,k] of drafter row (i,b,k)'s top-L tokens."""
+        target = np.ascontiguousarray(target)
+        drafter = np.ascontiguousarray(drafter)
+        assert target.dtype == drafter.dtype
+        N, B, P, V = drafter.shape
+        keep = np.ascontiguousarray(keep, dtype=np.int32)
+        assert keep.shape == (N, B, P)
+        alpha = np.empty((N, B, P), np.float64)
+        e_len = np.empty((N, B), np.float64)
+        if path is None:
+            assert target.shape == (B, P, V)
+            pp, M = None, 0
+        else:
+            pp = np.ascontiguousarray(path, dtype=np.int32)
+            M = target.shape[1]
+            assert target.shape == (B, M, V) and pp.shape == (B, P)
+        st = self.lib.orc_feedback_topl_pruned(_ptr(target), None if pp is None else _ptr(pp), M,
+                                               _ptr(drafter), dtype_code(target), N, B, P, V,
+                                               float(T), int(bool(greedy)), int(L), _ptr(keep),
+                                               _ptr(alpha), _ptr(e_len))
         return alpha, e_len, st
 
     # ---- learners ----------------------------------------------------------

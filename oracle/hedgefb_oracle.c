@@ -350,6 +350,88 @@ int orc_feedback_topl(const void* target, const int32_t* path, int M,
   return status;
 }
 
+/* ---- Thm 2 with EAGLE-2's dynamic pruning ------------------------------ */
+
+/* The remark closing Thm 2: when the draft tree is pruned, the candidate set
+ * of a node is its pruned set of children instead of Top_L(q).  A node's
+ * children are the drafter's L highest-ranked tokens and each is scored by
+ * the node's own score times q(child), so pruning by score keeps a prefix of
+ * that ranking: the first `keep` tokens of Top_L(q), 0 <= keep <= L (keep =
+ * 0: every child was pruned and the target's token cannot be accepted).
+ * alpha = sum over that prefix of p(v) (stochastic target) or 1[argmax p in
+ * the prefix] (greedy target).  keep outside [0, L] is an argument error
+ * (alpha NaN, ORC_BADARG); an unusable drafter or target row gives NaN and
+ * ORC_NONFINITE. */
+int orc_alpha_topl_pruned(const void* zt, const void* zd, int dtype, int V, double T,
+                          int greedy, int L, int keep, double* alpha) {
+  if (L < 1 || keep < 0 || keep > L) { *alpha = NAN; return ORC_BADARG; }
+  if (!row_ok(zd, dtype, V)) { *alpha = NAN; return ORC_NONFINITE; }
+  int n = L < V ? L : V;
+  int* idx = (int*)malloc(sizeof(int) * (size_t)n);
+  orc_topl_set(zd, dtype, V, n, idx);          /* Top_L(q), in rank order */
+  int kept = keep < n ? keep : n;             /* the pruned set: idx[0..kept-1] */
+  int st = ORC_OK;
+  if (greedy) {
+    int jt = orc_row_argmax(zt, dtype, V);
+    if (jt < 0) {
+      *alpha = NAN;
+      st = ORC_NONFINITE;
+    } else {
+      double a = 0.0;
+      for (int r = 0; r < kept; ++r)
+        if (idx[r] == jt) a = 1.0;
+      *alpha = a;
+    }
+  } else {
+    double* Pt = (double*)malloc(sizeof(double) * (size_t)V);
+    st = orc_row_probs(zt, dtype, V, T, Pt);
+    double a = 0.0;
+    for (int r = 0; r < kept; ++r) a += Pt[idx[r]];
+    *alpha = st ? NAN : a;
+    free(Pt);
+  }
+  free(idx);
+  return st;
+}
+
+/* A whole pruned-tree feedback call: as orc_feedback_topl, with keep[N,B,P]
+ * (element (i*B + b)*P + k) the number of children drafter i's tree kept at
+ * the node of position k of query b.  Returns ORC_BADARG if any keep is out
+ * of range (those alphas NaN), else ORC_NONFINITE if any row was unusable. */
+int orc_feedback_topl_pruned(const void* target, const int32_t* path, int M,
+                             const void* drafter, int dtype, int N, int B, int P,
+                             int V, double T, int greedy, int L, const int32_t* keep,
+                             double* alpha, double* e_len) {
+  if (N < 1 || B < 1 || P < 1 || V < 1 || L < 1 || (!greedy && !(T > 0.0)))
+    return ORC_BADARG;
+  if (path && M < 1) return ORC_BADARG;
+  size_t esz = (dtype == ORC_FP32) ? 4 : 2;
+  int bad_keep = 0, bad_row = 0;
+  for (int b = 0; b < B; ++b) {
+    for (int k = 0; k < P; ++k) {
+      if (path && (path[b * P + k] < 0 || path[b * P + k] >= M)) return ORC_BADARG;
+      const int64_t row_tgt = path ? (int64_t)b * M + path[b * P + k]  /* tree: path row */
+                                   : (int64_t)b * P + k;               /* chain: target[b, k] */
+      const char* zt = (const char*)target + (size_t)row_tgt * V * esz;
+      for (int i = 0; i < N; ++i) {
+        const int64_t row_drf = ((int64_t)i * B + b) * P + k;  /* drafter[i, b, k] */
+        const char* zd = (const char*)drafter + (size_t)row_drf * V * esz;
+        double a;
+        int st = orc_alpha_topl_pruned(zt, zd, dtype, V, T, greedy, L, keep[row_drf], &a);
+        if (st == ORC_BADARG) bad_keep = 1;
+        else if (st != ORC_OK) bad_row = 1;
+        alpha[row_drf] = a;
+      }
+    }
+  }
+  for (int i = 0; i < N; ++i)
+    for (int b = 0; b < B; ++b) {
+      const double* gam = alpha + ((size_t)i * B + b) * P;  /* alpha_1..alpha_K */
+      e_len[(size_t)i * B + b] = orc_elen_prefix(gam, P - 1);  /* Thm 3 */
+    }
+  return bad_keep ? ORC_BADARG : (bad_row ? ORC_NONFINITE : ORC_OK);
+}
+
 /* ---- learners ---------------------------------------------------------- */
 
 /* Hedge (App. B.1 remark): starting from w = 1, w_i <- w_i exp(-eta l_i)

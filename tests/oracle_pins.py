@@ -608,6 +608,134 @@ def check_feedback_topl_layout(o):
                 assert abs(e[i, b] - want_e) < 1e-12
 
 
+# ---- Thm 2 with EAGLE-2's dynamic pruning --------------------------------------
+
+def check_topl_pruned_prefix_scipy(o):
+    """Pruned candidate set = the first `keep` of the lexsort ranking: alpha
+    is scipy's softmax(z_t / T) summed over them (stochastic target), or
+    whether numpy's argmax of the target is among them (greedy target), for
+    every keep from 0 to L on tie-heavy rows with -inf masks."""
+    rng = np.random.default_rng(48)
+    for kind in KINDS:
+        for V in (3, 20, 300):
+            zt = stored(rng.normal(0, 2.5, V), kind)
+            zd = (rng.integers(-10, 10, V) / 4.0).astype(np.float32)
+            zd[rng.random(V) < 0.15] = -np.inf
+            zd = stored(zd, kind)
+            for L in (1, 4, 16):
+                rank = topl_numpy(zd, L)
+                for keep in range(L + 1):
+                    prefix = rank[:keep]
+                    for T in (0.6, 1.7):
+                        a, st = o.alpha_topl_pruned(zt, zd, T, False, L, keep)
+                        want = probs(zt, T)[prefix].sum()
+                        assert st == orc.OK and abs(a - want) < 1e-12, (kind, V, L, keep, T)
+                    a, st = o.alpha_topl_pruned(zt, zd, 1.0, True, L, keep)
+                    want = 1.0 if int(np.argmax(value(zt))) in set(prefix.tolist()) else 0.0
+                    assert st == orc.OK and a == want, (kind, V, L, keep)
+
+
+def check_topl_pruned_reductions(o):
+    """keep = L is the unpruned rule of Thm 2; keep = 1 under a greedy target
+    is the argmax-agreement rule; keep = 0 accepts nothing; alpha never
+    decreases as the pruning keeps more children."""
+    rng = np.random.default_rng(49)
+    for trial in range(60):
+        V = int(rng.integers(2, 60))
+        L = int(rng.integers(1, 17))
+        zt = stored(rng.normal(0, 2, V), "bf16")
+        zd = stored(value(zt) + rng.normal(0, 1.5, V), "bf16")
+        for greedy in (False, True):
+            a_full, st = o.alpha_topl(zt, zd, 0.9, greedy, L)
+            a, st2 = o.alpha_topl_pruned(zt, zd, 0.9, greedy, L, L)
+            assert st == st2 == orc.OK and a == a_full
+            a0, st = o.alpha_topl_pruned(zt, zd, 0.9, greedy, L, 0)
+            assert st == orc.OK and a0 == 0.0
+            prev = -1.0
+            for keep in range(L + 1):
+                a, st = o.alpha_topl_pruned(zt, zd, 0.9, greedy, L, keep)
+                assert st == orc.OK and a >= prev
+                prev = a
+        a, st = o.alpha_topl_pruned(zt, zd, 1.0, True, L, 1)
+        want = 1.0 if np.argmax(value(zt)) == np.argmax(value(zd)) else 0.0
+        assert st == orc.OK and a == want
+
+
+def check_topl_pruned_mc_eagle2(o):
+    """Monte Carlo of a pruned EAGLE-2 node on V = 8: the drafter expands its
+    L = 5 most likely tokens, scores each child by the node's score times
+    q(child), and drops the children scoring below a threshold; the target's
+    sampled token is accepted iff a surviving child matches it.  The
+    survivors are a prefix of the ranking, and the empirical acceptance rate
+    matches alpha with keep = their number, within 5 sigma."""
+    rng = np.random.default_rng(50)
+    V, n, L, T = 8, 400_000, 5, 0.8
+    zt = rng.normal(0, 1.5, V).astype(np.float32)
+    zd = rng.normal(0, 1.5, V).astype(np.float32)
+    q = softmax(zd.astype(np.float64))
+    children = np.argsort(-zd, kind="stable")[:L]
+    node_score = 0.6
+    scores = node_score * q[children]
+    threshold = np.sort(scores)[-3] * (1 - 1e-9)   # three children survive
+    survivors = children[scores >= threshold]
+    assert np.array_equal(survivors, children[:len(survivors)]), "pruning keeps a prefix"
+    x = rng.choice(V, size=n, p=probs(zt, T))
+    rate = np.isin(x, survivors).mean()
+    a, st = o.alpha_topl_pruned(zt, zd, T, False, L, len(survivors))
+    sigma = math.sqrt(a * (1 - a) / n)
+    assert st == orc.OK and len(survivors) == 3
+    assert abs(rate - a) < 5 * sigma + 1e-12, (rate, a, sigma)
+
+
+def check_topl_pruned_invalid(o):
+    """keep outside [0, L] is an argument error (NaN); unusable rows give
+    NaN and the non-finite status; a whole call reports the argument error
+    first and still fills every other alpha."""
+    rng = np.random.default_rng(51)
+    zt = rng.normal(0, 1, 30).astype(np.float32)
+    zd = rng.normal(0, 1, 30).astype(np.float32)
+    for keep in (-1, 5):
+        a, st = o.alpha_topl_pruned(zt, zd, 1.0, False, 4, keep)
+        assert st == orc.BADARG and np.isnan(a)
+    bad = zd.copy()
+    bad[2] = np.nan
+    a, st = o.alpha_topl_pruned(zt, bad, 1.0, False, 4, 2)
+    assert st == orc.NONFINITE and np.isnan(a)
+    N, B, P, V = 2, 2, 3, 30
+    tgt = stored(rng.normal(0, 2, (B, P, V)), "fp32")
+    drf = stored(rng.normal(0, 2, (N, B, P, V)), "fp32")
+    keep = rng.integers(0, 5, (N, B, P)).astype(np.int32)
+    keep[1, 0, 2] = 6
+    a, e, st = o.feedback_topl_pruned(tgt, drf, 1.0, False, 4, keep)
+    assert st == orc.BADARG and np.isnan(a[1, 0, 2]) and np.isnan(a).sum() == 1
+
+
+def check_feedback_topl_pruned_layout(o):
+    """The whole-call layout with per-row keep: alpha[i,b,k] pairs target row
+    (b,k) (or its path row) with drafter row (i,b,k) and that row's keep;
+    e_len is 1 + the sum of cumulative products of alpha_1..alpha_K."""
+    rng = np.random.default_rng(52)
+    N, B, P, V, L, T = 3, 2, 4, 40, 6, 0.9
+    tgt = stored(rng.normal(0, 2, (B, P, V)), "bf16")
+    drf = stored(value(tgt)[None] + rng.normal(0, 1, (N, B, P, V)), "bf16")
+    keep = rng.integers(0, L + 1, (N, B, P)).astype(np.int32)
+    M = 6
+    tree = stored(rng.normal(0, 2, (B, M, V)), "bf16")
+    path = rng.integers(0, M, (B, P)).astype(np.int32)
+    for use_path in (False, True):
+        a, e, st = o.feedback_topl_pruned(tree if use_path else tgt, drf, T, False, L, keep,
+                                          path if use_path else None)
+        assert st == orc.OK
+        for i in range(N):
+            for b in range(B):
+                for k in range(P):
+                    zt = tree[b, path[b, k]] if use_path else tgt[b, k]
+                    want = probs(zt, T)[topl_numpy(drf[i, b, k], L)[:keep[i, b, k]]].sum()
+                    assert abs(a[i, b, k] - want) < 1e-12
+                want_e = 1.0 + np.cumprod(a[i, b, :P - 1]).sum()
+                assert abs(e[i, b] - want_e) < 1e-12
+
+
 # ---- App. B.1 (QFI-D): sampled play --------------------------------------------
 
 def check_sample_select_searchsorted(o):

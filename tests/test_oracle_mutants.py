@@ -64,6 +64,17 @@ MUTANTS = {
                                       "const int64_t row_d = ((int64_t)b * N + i) * P + k;"),
     "topl_elen_all_positions": ("e_len[i * B + b] = orc_elen_prefix(gam, P - 1);",
                                 "e_len[i * B + b] = orc_elen_prefix(gam, P);"),
+    "pruned_ignores_keep": ("int kept = keep < n ? keep : n;", "int kept = n;"),
+    "pruned_keeps_one_more": ("int kept = keep < n ? keep : n;",
+                              "int kept = keep + 1 < n ? keep + 1 : n;"),
+    "pruned_keep_unchecked": ("if (L < 1 || keep < 0 || keep > L)", "if (L < 1)"),
+    "pruned_greedy_whole_set": ("for (int r = 0; r < kept; ++r)\n        if (idx[r] == jt) a = 1.0;",
+                                "for (int r = 0; r < n; ++r)\n        if (idx[r] == jt) a = 1.0;"),
+    "pruned_drafter_index_transposed": (
+        "const int64_t row_drf = ((int64_t)i * B + b) * P + k;",
+        "const int64_t row_drf = ((int64_t)b * N + i) * P + k;"),
+    "pruned_elen_all_positions": ("e_len[(size_t)i * B + b] = orc_elen_prefix(gam, P - 1);",
+                                  "e_len[(size_t)i * B + b] = orc_elen_prefix(gam, P);"),
     "hedge_state_not_cumulative": ("for (int i = 0; i < N; ++i) col[i] += f[i];",
                                    "for (int i = 0; i < N; ++i) col[i] = f[i];"),
     "sample_at_or_above": ("if (run > thr) return i;", "if (run >= thr) return i;"),
