@@ -177,8 +177,8 @@ int hs_feedback_topl_kernel_count(int N, int B, int P, int V);
  *                 L = 1 this is hs_feedback's greedy rule.
  *   workspace  device, hs_feedback_topl_workspace_size(...) bytes, 256-byte
  *              aligned (required).
- * The dynamic pruning of EAGLE-2 (Thm 2, last sentence) is not modelled:
- * the candidate set is the plain top L.  Errors as in hs_feedback; a
+ * The candidate set is the plain top L; hs_feedback_topl_pruned below takes
+ * the pruned sets of EAGLE-2's dynamic pruning.  Errors as in hs_feedback; a
  * drafter row with NaN, +inf or no finite logit gives NaN and
  * HS_ERR_NONFINITE. */
 hs_status hs_feedback_topl(const void* target, const void* drafter, int dtype, int N,
@@ -194,6 +194,36 @@ hs_status hs_feedback_topl_path(const void* tree_target, const int32_t* path_idx
                                 float* alpha, float* e_len, void* workspace,
                                 size_t workspace_bytes, int* dev_status,
                                 void* stream);
+
+/* Tree-mode feedback with EAGLE-2's dynamic pruning (Sec. 2.3, the remark
+ * closing Thm 2: with pruning, the candidate set of a node is its pruned set
+ * of children).  A node's children are the drafter's L highest-ranked tokens
+ * and each is scored by the node's score times q(child), so pruning by score
+ * keeps a prefix of that ranking.  Same arguments as hs_feedback_topl, plus
+ *   keep  device, [N,B,P] int32, caller-owned: keep[i,b,k] in [0, L] is the
+ *         number of children drafter i's tree kept at the node of position k
+ *         of query b; the candidate set is the first keep[i,b,k] tokens of
+ *         Top_L(q_i) (0: every child was pruned, alpha = 0).  keep = L
+ *         everywhere gives hs_feedback_topl's result.  Must be non-null and
+ *         4-byte aligned (HS_ERR_INVALID_ARG / HS_ERR_MISALIGNED before any
+ *         launch).  A value outside [0, L] makes that alpha NaN and stores
+ *         HS_ERR_INVALID_ARG to *dev_status.
+ * Workspace: hs_feedback_topl_workspace_size(N, B, P, V); launches:
+ * hs_feedback_topl_kernel_count(N, B, P, V). */
+hs_status hs_feedback_topl_pruned(const void* target, const void* drafter, int dtype, int N,
+                                  int B, int P, int V, float temperature, int greedy, int L,
+                                  const int32_t* keep, float* alpha, float* e_len,
+                                  void* workspace, size_t workspace_bytes, int* dev_status,
+                                  void* stream);
+
+/* hs_feedback_topl_pruned with the target rows taken from a draft tree, as
+ * in hs_feedback_path (tree_target [B,M,V], path_idx [B,P] int32). */
+hs_status hs_feedback_topl_pruned_path(const void* tree_target, const int32_t* path_idx,
+                                       int M, const void* drafter, int dtype, int N, int B,
+                                       int P, int V, float temperature, int greedy, int L,
+                                       const int32_t* keep, float* alpha, float* e_len,
+                                       void* workspace, size_t workspace_bytes,
+                                       int* dev_status, void* stream);
 
 /* Hedge weights from cumulative losses (App. B.1 remark: w_i <- w_i
  * exp(-eta l_i) from w = 1, normalised, i.e. w = exp(-eta L) / Z).
@@ -370,6 +400,26 @@ typedef struct {
 
 hs_status hs_schedule_next(const hs_schedule_config* cfg, hs_schedule_state* state,
                            int tokens, hs_schedule_action* action);
+
+/* ---- test hook (the paper has no counterpart) ----------------------------
+ * Exercises the bounded-wait error path of the library's kernels on a GPU
+ * without faulting or hanging it.  It runs the streaming stochastic kernel
+ * (the one hs_feedback uses for V > 153 600) with one change: the wait of
+ * tile (b,k) = (0,0) for its statistics asks for one chunk more than exist,
+ * so it can only run out, and every wait is limited to `wait_cycles` SM clock
+ * cycles instead of about a second.  Tile (0,0)'s waits then report
+ * HS_ERR_TIMEOUT to *dev_status and its alphas (and the e_len of query 0)
+ * come out NaN; every other alpha is the one hs_feedback computes, and the
+ * CUDA context stays usable.  Same arguments as hs_feedback (stochastic,
+ * chain target), plus wait_cycles >= 1; dev_status is required.  Takes only
+ * shapes the streaming kernel takes (bf16/fp16, V % 8 == 0, N <= 32,
+ * 16-byte-aligned logits), else HS_ERR_UNSUPPORTED; workspace as
+ * hs_feedback_workspace_size reports for the same sizes. */
+hs_status hs_test_stream_wait_timeout(const void* target, const void* drafter, int dtype,
+                                      int N, int B, int P, int V, float temperature,
+                                      long long wait_cycles, float* alpha, float* e_len,
+                                      void* workspace, size_t workspace_bytes,
+                                      int* dev_status, void* stream);
 
 #ifdef __cplusplus
 }

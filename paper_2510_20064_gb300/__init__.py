@@ -38,11 +38,17 @@ SIGNATURES = {
     "hs_feedback": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_static": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _P, _P, _P, _P], _I),
+    "hs_test_stream_wait_timeout": ([_P, _P, _I, _I, _I, _I, _I, _F, ctypes.c_longlong, _P, _P, _P,
+                                     _Z, _P, _P], _I),
     "hs_feedback_topl_workspace_size": ([_I, _I, _I, _I], _Z),
     "hs_feedback_topl_kernel_count": ([_I, _I, _I, _I], _I),
     "hs_feedback_topl": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z, _P, _P], _I),
     "hs_feedback_topl_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _Z,
                                _P, _P], _I),
+    "hs_feedback_topl_pruned": ([_P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P, _P, _Z, _P,
+                                 _P], _I),
+    "hs_feedback_topl_pruned_path": ([_P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P, _P, _P,
+                                      _P, _Z, _P, _P], _I),
     "hs_hedge_update": ([_P, _I, _I, _F, _P, _P, _P], _I),
     "hs_normalhedge_update": ([_P, _P, _P, _I, _I, _P, _P], _I),
     "hs_learner_step": ([_P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P], _I),
@@ -256,6 +262,49 @@ def hs_feedback_topl_path(tree_target: torch.Tensor, path_idx: torch.Tensor,
                                      int(bool(greedy)), int(L), _ptr(alpha), _ptr(e_len),
                                      _ptr(workspace), ws_bytes, _ptr(dev_status), _stream(stream))
     _check(st, "hs_feedback_topl_path")
+    return alpha, e_len
+
+
+def hs_feedback_topl_pruned(target: torch.Tensor, drafter: torch.Tensor, L: int,
+                            keep: torch.Tensor, temperature: float = 1.0, greedy: bool = False,
+                            alpha=None, e_len=None, workspace=None, dev_status=None,
+                            stream=None):
+    """Draft-tree feedback with dynamically pruned child sets (the remark
+    closing Thm 2): drafter row (i,b,k)'s candidates are the first
+    keep[i,b,k] (int32 [N,B,P], 0..L) of its top-L tokens."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(target, "target", drafter.dtype, (B, P, V))
+    _need(keep, "keep", torch.int32, (N, B, P))
+    alpha, e_len, workspace, ws_bytes = _topl_outputs(drafter, alpha, e_len, workspace)
+    st = lib().hs_feedback_topl_pruned(_ptr(target), _ptr(drafter), _dtype_code(drafter), N, B, P,
+                                       V, float(temperature), int(bool(greedy)), int(L),
+                                       _ptr(keep), _ptr(alpha), _ptr(e_len), _ptr(workspace),
+                                       ws_bytes, _ptr(dev_status), _stream(stream))
+    _check(st, "hs_feedback_topl_pruned")
+    return alpha, e_len
+
+
+def hs_feedback_topl_pruned_path(tree_target: torch.Tensor, path_idx: torch.Tensor,
+                                 drafter: torch.Tensor, L: int, keep: torch.Tensor,
+                                 temperature: float = 1.0, greedy: bool = False, alpha=None,
+                                 e_len=None, workspace=None, dev_status=None, stream=None):
+    """As hs_feedback_topl_pruned with target row (b,k) = tree_target[b, path_idx[b,k]]."""
+    _need(drafter, "drafter")
+    N, B, P, V = drafter.shape
+    _need(tree_target, "tree_target", drafter.dtype)
+    if tree_target.dim() != 3 or tree_target.shape[0] != B or tree_target.shape[2] != V:
+        raise ValueError(f"tree_target must be [B, M, V] = [{B}, M, {V}]")
+    M = tree_target.shape[1]
+    _need(path_idx, "path_idx", torch.int32, (B, P))
+    _need(keep, "keep", torch.int32, (N, B, P))
+    alpha, e_len, workspace, ws_bytes = _topl_outputs(drafter, alpha, e_len, workspace)
+    st = lib().hs_feedback_topl_pruned_path(_ptr(tree_target), _ptr(path_idx), M, _ptr(drafter),
+                                            _dtype_code(drafter), N, B, P, V, float(temperature),
+                                            int(bool(greedy)), int(L), _ptr(keep), _ptr(alpha),
+                                            _ptr(e_len), _ptr(workspace), ws_bytes,
+                                            _ptr(dev_status), _stream(stream))
+    _check(st, "hs_feedback_topl_pruned_path")
     return alpha, e_len
 
 

@@ -338,8 +338,8 @@ hs_status feedback_common(const void* target, const int32_t* path, int M, const 
 // Draft-tree feedback (Thm 2): validation shared by the chain and path entries.
 hs_status topl_common(const void* target, const int32_t* path, int M, const void* drafter,
                       int dtype, int N, int B, int P, int V, float temperature, int greedy, int L,
-                      float* alpha, float* e_len, void* ws, size_t ws_bytes, int* dev_status,
-                      void* stream) {
+                      const int32_t* keep, float* alpha, float* e_len, void* ws, size_t ws_bytes,
+                      int* dev_status, void* stream) {
   if (dtype != HS_BF16 && dtype != HS_FP16 && dtype != HS_FP32) return HS_ERR_INVALID_ARG;
   if (!sizes_ok(N, B, P, V)) return HS_ERR_INVALID_ARG;
   if (L < 1) return HS_ERR_INVALID_ARG;
@@ -350,13 +350,13 @@ hs_status topl_common(const void* target, const int32_t* path, int M, const void
   const int esz = elem_bytes(dtype);
   if (reinterpret_cast<uintptr_t>(target) % esz || reinterpret_cast<uintptr_t>(drafter) % esz ||
       reinterpret_cast<uintptr_t>(alpha) % 4 || reinterpret_cast<uintptr_t>(e_len) % 4 ||
-      reinterpret_cast<uintptr_t>(dev_status) % 4)
+      reinterpret_cast<uintptr_t>(dev_status) % 4 || reinterpret_cast<uintptr_t>(keep) % 4)
     return HS_ERR_MISALIGNED;
   if (!ws || ws_bytes < topl::workspace_bytes(N, B, P, V)) return HS_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(ws) % 256) return HS_ERR_MISALIGNED;
   const float c = kLog2e / (greedy ? 1.f : temperature);
-  return topl::launch(target, path, M, drafter, dtype, N, B, P, V, L, greedy, c, alpha, e_len, ws,
-                      dev_status, static_cast<cudaStream_t>(stream));
+  return topl::launch(target, path, M, drafter, dtype, N, B, P, V, L, keep, greedy, c, alpha,
+                      e_len, ws, dev_status, static_cast<cudaStream_t>(stream));
 }
 
 }  // namespace
@@ -377,7 +377,18 @@ extern "C" hs_status hs_feedback_topl(const void* target, const void* drafter, i
                                       float* alpha, float* e_len, void* workspace,
                                       size_t workspace_bytes, int* dev_status, void* stream) {
   return hs::topl_common(target, nullptr, 0, drafter, dtype, N, B, P, V, temperature, greedy, L,
-                         alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+                         nullptr, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" hs_status hs_feedback_topl_pruned(const void* target, const void* drafter, int dtype,
+                                             int N, int B, int P, int V, float temperature,
+                                             int greedy, int L, const int32_t* keep, float* alpha,
+                                             float* e_len, void* workspace,
+                                             size_t workspace_bytes, int* dev_status,
+                                             void* stream) {
+  if (!keep) return HS_ERR_INVALID_ARG;
+  return hs::topl_common(target, nullptr, 0, drafter, dtype, N, B, P, V, temperature, greedy, L,
+                         keep, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
 }
 
 extern "C" hs_status hs_feedback_topl_path(const void* tree_target, const int32_t* path_idx,
@@ -390,7 +401,24 @@ extern "C" hs_status hs_feedback_topl_path(const void* tree_target, const int32_
   if (reinterpret_cast<uintptr_t>(path_idx) % 4) return HS_ERR_MISALIGNED;
   if (double(B) * double(M) * double(V) >= 4.6e18) return HS_ERR_INVALID_ARG;
   return hs::topl_common(tree_target, path_idx, M, drafter, dtype, N, B, P, V, temperature,
-                         greedy, L, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+                         greedy, L, nullptr, alpha, e_len, workspace, workspace_bytes, dev_status,
+                         stream);
+}
+
+extern "C" hs_status hs_feedback_topl_pruned_path(const void* tree_target,
+                                                  const int32_t* path_idx, int M,
+                                                  const void* drafter, int dtype, int N, int B,
+                                                  int P, int V, float temperature, int greedy,
+                                                  int L, const int32_t* keep, float* alpha,
+                                                  float* e_len, void* workspace,
+                                                  size_t workspace_bytes, int* dev_status,
+                                                  void* stream) {
+  if (!path_idx || M < 1 || !keep) return HS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(path_idx) % 4) return HS_ERR_MISALIGNED;
+  if (double(B) * double(M) * double(V) >= 4.6e18) return HS_ERR_INVALID_ARG;
+  return hs::topl_common(tree_target, path_idx, M, drafter, dtype, N, B, P, V, temperature,
+                         greedy, L, keep, alpha, e_len, workspace, workspace_bytes, dev_status,
+                         stream);
 }
 
 extern "C" size_t hs_feedback_workspace_size(int N, int B, int P, int V, int dtype, int greedy) {
@@ -425,4 +453,24 @@ extern "C" hs_status hs_feedback_path(const void* tree_target, const int32_t* pa
   if (double(B) * double(M) * double(V) >= 4.6e18) return HS_ERR_INVALID_ARG;
   return hs::feedback_common(tree_target, path_idx, M, drafter, dtype, N, B, P, V, temperature,
                              greedy, alpha, e_len, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" hs_status hs_test_stream_wait_timeout(const void* target, const void* drafter,
+                                                 int dtype, int N, int B, int P, int V,
+                                                 float temperature, long long wait_cycles,
+                                                 float* alpha, float* e_len, void* workspace,
+                                                 size_t workspace_bytes, int* dev_status,
+                                                 void* stream) {
+  if (!hs::sizes_ok(N, B, P, V) || !target || !drafter || !alpha || !dev_status)
+    return HS_ERR_INVALID_ARG;
+  if (!(isfinite(temperature) && temperature > 0.f) || wait_cycles < 1) return HS_ERR_INVALID_ARG;
+  if (!hs::stream::eligible(target, drafter, dtype, N, V, 0)) return HS_ERR_UNSUPPORTED;
+  if (reinterpret_cast<uintptr_t>(alpha) % 4 || reinterpret_cast<uintptr_t>(e_len) % 4 ||
+      reinterpret_cast<uintptr_t>(dev_status) % 4 || reinterpret_cast<uintptr_t>(workspace) % 256)
+    return HS_ERR_MISALIGNED;
+  if (!workspace || workspace_bytes < hs::stream::workspace_bytes(N, B, P, V))
+    return HS_ERR_INVALID_ARG;
+  return hs::stream::launch_wait_test(target, drafter, dtype, N, B, P, V, hs::kLog2e / temperature,
+                                      wait_cycles, alpha, e_len, workspace, dev_status,
+                                      static_cast<cudaStream_t>(stream));
 }

@@ -18,8 +18,9 @@
 //     and writes alpha[:, b, k].
 // No overlap ever waits on a later item than the ones its own CTA has
 // already passed, and the launch is cooperative (all CTAs resident), so the
-// waits always end; each is bounded anyway (HS_ERR_TIMEOUT).  HBM traffic is
-// one read of every logit; L2 traffic two.
+// waits always end; each is bounded anyway: a wait that gives up reports
+// HS_ERR_TIMEOUT and marks its tile, whose alphas are then written as NaN.
+// HBM traffic is one read of every logit; L2 traffic two.
 #include <math.h>
 #include <stdint.h>
 
@@ -38,6 +39,9 @@ constexpr int kVecs = 4;                         // 16-byte vectors per thread a
 constexpr int kChunk = kThreads * kVecs * 8;     // logits per row chunk (bf16 / fp16)
 constexpr int kMaxN = 32;
 constexpr long long kTimeoutCycles = 1LL << 31;  // about a second
+// A tile's overlap count carries this mark once an overlap of the tile gave
+// up waiting for the tile's statistics (chunks per row stay below it).
+constexpr int kTimedOut = 1 << 24;
 
 struct Params {
   const void* target;
@@ -56,6 +60,8 @@ struct Params {
   int* cnt2;      // [ntiles] chunks with overlap
   float* alpha;
   int* dev_status;
+  long long wait_limit;  // clock cycles a wait may take (kTimeoutCycles)
+  int stall_tile;        // test hook: this tile's statistics count never completes (-1: none)
 };
 
 // Order-preserving int key of a float (NaN above +inf): warp max in one redux.
@@ -137,6 +143,7 @@ struct Smem {
   float2 os[kMaxN + 1];           // row (offset O, 1/Z) of the overlap item
   float ap[kMaxN][kWarps];        // per-warp alpha partials
   int flag;                       // 1: this CTA finishes the tile's alpha
+  int wait_mark;                  // kTimedOut when this overlap's wait gave up
 };
 
 template <int DT>
@@ -192,21 +199,26 @@ __device__ void overlap_item(const Params& p, Smem& sm, int y) {
   const int j = y % p.nchunk;
   const int R = p.N + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // every chunk of tile t has its stats (bounded wait)
+  // every chunk of tile t has its stats (bounded wait; the test hook asks
+  // for one chunk more than exist, so that the wait runs out)
   if (threadIdx.x == 0) {
+    const int need = p.nchunk + (t == p.stall_tile ? 1 : 0);
     const long long t0 = clock64();
     int seen;
+    sm.wait_mark = 0;
     while (true) {
       asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(seen) : "l"(p.cnt + t) : "memory");
-      if (seen >= p.nchunk) break;
-      if (clock64() - t0 > kTimeoutCycles) {
+      if (seen >= need) break;
+      if (clock64() - t0 > p.wait_limit) {
         report(p.dev_status, HS_ERR_TIMEOUT);
+        sm.wait_mark = kTimedOut;
         break;
       }
       __nanosleep(64);
     }
   }
   __syncthreads();
+  const int mark = sm.wait_mark;  // rewritten only after this call's later barriers
   // row offsets and normalisers: warp w merges rows w, w + kWarps, ...
   for (int r = warp; r < R; r += kWarps) {
     float o = -INFINITY, s = 0.f;
@@ -269,19 +281,29 @@ __device__ void overlap_item(const Params& p, Smem& sm, int y) {
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
-    sm.flag = atomicAdd(p.cnt2 + t, 1) == p.nchunk - 1;
+    // the count of finished overlaps (low bits) and the mark of a wait that
+    // gave up (one bit, set before this CTA's count: the tile's last count
+    // sees every mark)
+    if (mark) atomicOr(p.cnt2 + t, kTimedOut);
+    const int before = atomicAdd(p.cnt2 + t, 1);
+    sm.flag = ((before & (kTimedOut - 1)) == p.nchunk - 1) ? 1 + ((before | mark) & kTimedOut)
+                                                           : 0;
     __threadfence();
   }
   __syncthreads();
   if (!sm.flag) return;
-  // this CTA completed tile t: alpha[:, b, k] from the chunk partials
+  // this CTA completed tile t: alpha[:, b, k] from the chunk partials (NaN
+  // when one of the tile's waits gave up)
+  const bool timed_out = (sm.flag & kTimedOut) != 0;
   const int64_t b = t / p.P, k = t % p.P;
   const bool bad_path = p.path && (p.path[t] < 0 || p.path[t] >= p.M);
   const bool t_ok = !isnan(sm.os[0].x);
   for (int i = threadIdx.x; i < p.N; i += kThreads) {
     float a = 0.f;
     for (int q = 0; q < p.nchunk; ++q) a += __ldcg(p.apart + (t * p.N + i) * p.nchunk + q);
-    if (bad_path || !t_ok || isnan(sm.os[i + 1].x)) {
+    if (timed_out) {
+      a = __int_as_float(0x7fc00000);
+    } else if (bad_path || !t_ok || isnan(sm.os[i + 1].x)) {
       a = __int_as_float(0x7fc00000);
       report(p.dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
     }
@@ -403,9 +425,10 @@ bool eligible(const void* target, const void* drafter, int dtype, int N, int V, 
 
 size_t workspace_bytes(int N, int B, int P, int V) { return layout(N, B, P, V).total; }
 
-hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
-                 int N, int B, int P, int V, float c, float* alpha, float* e_len, void* ws,
-                 int* dev_status, cudaStream_t stream) {
+hs_status launch_impl(const void* target, const int32_t* path, int M, const void* drafter,
+                      int dtype, int N, int B, int P, int V, float c, float* alpha, float* e_len,
+                      void* ws, int* dev_status, cudaStream_t stream, int stall_tile,
+                      long long wait_limit) {
   Params p = {};
   p.target = target;
   p.path = path;
@@ -422,6 +445,8 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   p.lag = 1;
   p.alpha = alpha;
   p.dev_status = dev_status;
+  p.stall_tile = stall_tile;
+  p.wait_limit = wait_limit;
   const hs_status st = dtype == HS_BF16 ? launch_t<HS_BF16>(p, ws, stream)
                                         : launch_t<HS_FP16>(p, ws, stream);
   if (st != HS_OK) return st;
@@ -432,6 +457,20 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
       return HS_ERR_CUDA;
   }
   return HS_OK;
+}
+
+hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
+                 int N, int B, int P, int V, float c, float* alpha, float* e_len, void* ws,
+                 int* dev_status, cudaStream_t stream) {
+  return launch_impl(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, ws, dev_status,
+                     stream, -1, kTimeoutCycles);
+}
+
+hs_status launch_wait_test(const void* target, const void* drafter, int dtype, int N, int B,
+                           int P, int V, float c, long long wait_cycles, float* alpha,
+                           float* e_len, void* ws, int* dev_status, cudaStream_t stream) {
+  return launch_impl(target, nullptr, 0, drafter, dtype, N, B, P, V, c, alpha, e_len, ws,
+                     dev_status, stream, 0, wait_cycles);
 }
 
 }  // namespace stream

@@ -27,5 +27,14 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
                  int N, int B, int P, int V, float c, float* alpha, float* e_len, void* ws,
                  int* dev_status, cudaStream_t stream);
 
+// Test hook for the bounded waits: launch() with tile 0's statistics count
+// made unreachable (one chunk more is awaited than exist) and every wait
+// limited to wait_cycles clock cycles, so that tile 0's waits run out: they
+// report HS_ERR_TIMEOUT and tile 0's alphas are written as NaN, while every
+// other tile completes normally.
+hs_status launch_wait_test(const void* target, const void* drafter, int dtype, int N, int B,
+                           int P, int V, float c, long long wait_cycles, float* alpha,
+                           float* e_len, void* ws, int* dev_status, cudaStream_t stream);
+
 }  // namespace stream
 }  // namespace hs

@@ -18,7 +18,8 @@
 //                 several steps in flight without holding them in registers.
 //   alpha_kernel  one warp per drafter row: merges the N S target partials of
 //                 its (b, k) and the S key lists of its row, and sums p over
-//                 the row's top L (greedy target: compares with the first
+//                 the row's top L, or over the first keep[row] of them when
+//                 the tree was pruned (greedy target: compares with the first
 //                 argmax); the last warp of each (i, b) to finish forms e_len.
 // Every logit is read once.  The ranking is by the stored drafter logits
 // (q's order does not depend on the temperature), ties toward the lower
@@ -59,6 +60,7 @@ struct Params {
   TStat* stats;      // [B*P][N*S]
   uint64_t* parts;   // [N*B*P][S][kPartSlots]
   int* counters;     // [N*B] warps done per (i, b), for e_len
+  const int32_t* keep;  // [N*B*P] children kept by the tree's pruning, or null (all L)
   float* alpha;
   float* e_len;
   int* dev_status;
@@ -584,10 +586,18 @@ __global__ void __launch_bounds__(kThreads) alpha_kernel(const Params p) {
       if (l == q) key = best;
     }
   }
+  // the candidate set: the first `kept` of the row's L ranked keys (Thm 2's
+  // remark on pruning: a pruned node keeps a prefix of its children)
+  int kept = p.L;
+  bool keep_bad = false;
+  if (p.keep) {
+    kept = __ldg(p.keep + r);
+    keep_bad = kept < 0 || kept > p.L;
+  }
   const bool target_ok =
       flags == 0 && gm != -INFINITY && (p.greedy || (isfinite(s) && s > 0.f));
-  const bool ok = !(f & 1ull) && (f & 2ull) && target_ok;
-  const int mine = (l < p.L && key != 0ull) ? int(0xffffffffu - uint32_t(key)) : -1;
+  const bool ok = !(f & 1ull) && (f & 2ull) && target_ok && !keep_bad;
+  const int mine = (l < kept && key != 0ull) ? int(0xffffffffu - uint32_t(key)) : -1;
   float a = 0.f;
   if (ok && mine >= 0) {
     if (p.greedy) {
@@ -603,7 +613,7 @@ __global__ void __launch_bounds__(kThreads) alpha_kernel(const Params p) {
   if (l == 0) {
     if (!ok) {
       a = __int_as_float(0x7fc00000);
-      report(p.dev_status, (flags & 2) ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
+      report(p.dev_status, (keep_bad || (flags & 2)) ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
     }
     p.alpha[r] = a;
     if (p.e_len) {
@@ -676,8 +686,8 @@ size_t workspace_bytes(int N, int B, int P, int V) {
 }
 
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
-                 int N, int B, int P, int V, int L, int greedy, float c, float* alpha,
-                 float* e_len, void* ws, int* dev_status, cudaStream_t stream) {
+                 int N, int B, int P, int V, int L, const int32_t* keep, int greedy, float c,
+                 float* alpha, float* e_len, void* ws, int* dev_status, cudaStream_t stream) {
   const int esz = dtype == HS_FP32 ? 4 : 2;
   const bool vec = (int64_t(V) * esz) % 16 == 0 && reinterpret_cast<uintptr_t>(target) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(drafter) % 16 == 0;
@@ -692,6 +702,7 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   p.P = P;
   p.V = V;
   p.L = L;
+  p.keep = keep;
   p.S = split_of(p.nrows, V);
   p.greedy = greedy;
   p.c = c;

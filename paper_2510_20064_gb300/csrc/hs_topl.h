@@ -20,10 +20,13 @@ size_t workspace_bytes(int N, int B, int P, int V);
 // Kernels one launch() runs.
 int kernel_count(int N, int B, int P, int V);
 
-// alpha [N,B,P] (and e_len [N,B] when non-null); c = log2(e) / T.
+// alpha [N,B,P] (and e_len [N,B] when non-null); c = log2(e) / T.  keep
+// (device [N,B,P] int32, or null for all L): the candidate set of drafter row
+// r is the first keep[r] tokens of its top L; a keep outside [0, L] gives NaN
+// and HS_ERR_INVALID_ARG in *dev_status.
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
-                 int N, int B, int P, int V, int L, int greedy, float c, float* alpha,
-                 float* e_len, void* ws, int* dev_status, cudaStream_t stream);
+                 int N, int B, int P, int V, int L, const int32_t* keep, int greedy, float c,
+                 float* alpha, float* e_len, void* ws, int* dev_status, cudaStream_t stream);
 
 }  // namespace topl
 }  // namespace hs

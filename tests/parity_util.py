@@ -63,22 +63,24 @@ def host_threads() -> int:
         return os.cpu_count() or 1
 
 
-def oracle_feedback_parallel(d: dict, T: float, greedy: bool):
-    """oracle_feedback on every host core: the queries are independent, so
-    each thread runs the oracle on one query's rows (its own contiguous copy)
-    and the results are stacked in query order.  Same arithmetic, same
-    outputs as one oracle call over all queries."""
-    o = oracle.get()
+def per_query_parallel(call, d: dict, keep: np.ndarray | None = None):
+    """Run a whole-call oracle function on every host core: the queries are
+    independent, so each thread calls `call(target, drafter, path[, keep])`
+    on one query's rows (contiguous copies) and the results are stacked in
+    query order -- the same arithmetic and outputs as one call over all
+    queries.  Returns (alpha, e_len, first non-zero status or 0)."""
     t_np = synth.storage_numpy(d["target"])
     d_np = synth.storage_numpy(d["drafter"])
     path = d.get("path")
     path_np = None if path is None else path.cpu().numpy().astype(np.int32)
-    N, B, P, V = d_np.shape
+    B = d_np.shape[1]
 
     def one(b):
-        pb = None if path_np is None else np.ascontiguousarray(path_np[b:b + 1])
-        return o.feedback(np.ascontiguousarray(t_np[b:b + 1]),
-                          np.ascontiguousarray(d_np[:, b:b + 1]), T, greedy, path=pb)
+        args = [np.ascontiguousarray(t_np[b:b + 1]), np.ascontiguousarray(d_np[:, b:b + 1]),
+                None if path_np is None else np.ascontiguousarray(path_np[b:b + 1])]
+        if keep is not None:
+            args.append(np.ascontiguousarray(keep[:, b:b + 1]))
+        return call(*args)
 
     with cf.ThreadPoolExecutor(max_workers=host_threads()) as ex:
         parts = list(ex.map(one, range(B)))
@@ -86,3 +88,9 @@ def oracle_feedback_parallel(d: dict, T: float, greedy: bool):
     e_len = np.concatenate([e for _, e, _ in parts], axis=1)
     status = next((st for _, _, st in parts if st != 0), 0)
     return alpha, e_len, status
+
+
+def oracle_feedback_parallel(d: dict, T: float, greedy: bool):
+    """oracle_feedback on every host core (per_query_parallel)."""
+    o = oracle.get()
+    return per_query_parallel(lambda t, dr, pa: o.feedback(t, dr, T, greedy, path=pa), d)

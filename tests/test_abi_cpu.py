@@ -188,3 +188,36 @@ def test_binding_refuses_cpu_tensors(hf):
     t = torch.zeros(1, 3, 8)
     with pytest.raises(ValueError):
         hf.hs_feedback(t, torch.zeros(2, 1, 3, 8))
+
+
+def test_pruned_tree_entries_reject_bad_keep(hf):
+    """The pruned tree-mode entries refuse a null or misaligned kept-count
+    array before anything reaches the GPU."""
+    lib = hf.lib()
+    P = ctypes.c_void_p
+    for keep, want in ((None, hf.HS_ERR_INVALID_ARG), (P(FAKE + 2), hf.HS_ERR_MISALIGNED)):
+        st = lib.hs_feedback_topl_pruned(P(FAKE), P(FAKE), hf.HS_BF16, 2, 2, 3, 64, 1.0, 0, 4,
+                                         keep, P(FAKE), P(FAKE), P(FAKE), 1 << 20, None, None)
+        assert st == want
+        st = lib.hs_feedback_topl_pruned_path(P(FAKE), P(FAKE), 5, P(FAKE), hf.HS_BF16, 2, 2, 3,
+                                              64, 1.0, 0, 4, keep, P(FAKE), P(FAKE), P(FAKE),
+                                              1 << 20, None, None)
+        assert st == want
+
+
+def test_wait_timeout_hook_refuses_other_shapes(hf):
+    """The bounded-wait test hook takes only the streaming kernel's shapes
+    and a positive limit, and needs the status word; anything else is
+    refused before anything reaches the GPU."""
+    lib = hf.lib()
+    fake = ctypes.c_void_p(FAKE)
+    lim = ctypes.c_longlong
+    assert lib.hs_test_stream_wait_timeout(fake, fake, hf.HS_FP32, 2, 1, 2, 200000, 1.0,
+                                           lim(1000), fake, fake, fake, 1 << 30, fake,
+                                           None) == hf.HS_ERR_UNSUPPORTED
+    assert lib.hs_test_stream_wait_timeout(fake, fake, hf.HS_BF16, 2, 1, 2, 200000, 1.0,
+                                           lim(0), fake, fake, fake, 1 << 30, fake,
+                                           None) == hf.HS_ERR_INVALID_ARG
+    assert lib.hs_test_stream_wait_timeout(fake, fake, hf.HS_BF16, 2, 1, 2, 200000, 1.0,
+                                           lim(1000), fake, fake, fake, 1 << 30, None,
+                                           None) == hf.HS_ERR_INVALID_ARG

@@ -12,7 +12,7 @@ import torch
 import oracle
 import paper_2510_20064_gb300 as hf
 from paper_2510_20064_gb300 import synth
-from parity_util import RTOL_ALPHA, assert_rel, to_np
+from parity_util import RTOL_ALPHA, assert_rel, per_query_parallel, to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -172,3 +172,88 @@ def test_topl_full_size_sampled(name):
                 assert a[i, b, k] == ra
             else:
                 assert abs(a[i, b, k] - ra) <= RTOL_ALPHA * abs(ra), (i, b, k, a[i, b, k], ra)
+
+
+# ---- EAGLE-2's dynamic pruning (the remark closing Thm 2) ----------------------
+
+def run_pruned(d, T, greedy, L, keep):
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    kt = torch.tensor(keep, dtype=torch.int32, device=DEV)
+    if "path" in d:
+        a, e = hf.hs_feedback_topl_pruned_path(d["target"], d["path"], d["drafter"], L, kt, T,
+                                               greedy, dev_status=status)
+    else:
+        a, e = hf.hs_feedback_topl_pruned(d["target"], d["drafter"], L, kt, T, greedy,
+                                          dev_status=status)
+    torch.cuda.synchronize()
+    return to_np(a), to_np(e), int(status.item())
+
+
+def oracle_pruned(d, T, greedy, L, keep):
+    o = oracle.get()
+    return per_query_parallel(
+        lambda t, dr, pa, kp: o.feedback_topl_pruned(t, dr, T, greedy, L, kp, path=pa), d, keep)
+
+
+PRUNED = [
+    ("qwen3_8b_chain", dict(B=2, N=3, P=3), (1, 4, 10, 16)),
+    ("tree_path", dict(B=2, N=3), (1, 4, 10, 16)),
+    ("tree_path", {}, (10,)),  # the full tree_path call: 2048 rows, one warp each
+]
+
+
+@pytest.mark.parametrize("name,sizes,L", [(n, s, L) for n, s, Ls in PRUNED for L in Ls],
+                         ids=[f"{n}{'_full' if not s else ''}_L{L}" for n, s, Ls in PRUNED
+                              for L in Ls])
+def test_pruned_matches_oracle(name, sizes, L):
+    """Per-row kept-children counts drawn from 0..L (every value occurs):
+    every alpha and e_len against the oracle; the candidate sets are exact."""
+    w = W[name]
+    d = synth.make_inputs(w, device=DEV, seed=800 + L, **sizes)
+    N, B, P = d["drafter"].shape[:3]
+    rng = np.random.default_rng(900 + L)
+    keep = rng.integers(0, L + 1, (N, B, P)).astype(np.int32)
+    keep.reshape(-1)[:L + 1] = np.arange(L + 1)
+    for greedy in (False, True):
+        a, e, st = run_pruned(d, w.temperature, greedy, L, keep)
+        ra, re, rst = oracle_pruned(d, w.temperature, greedy, L, keep)
+        assert st == hf.HS_OK and rst == 0, (st, rst)
+        if greedy:
+            assert np.array_equal(a, ra) and np.array_equal(e, re)
+        else:
+            assert_rel(a, ra, RTOL_ALPHA, f"pruned alpha L={L}")
+            assert_rel(e, re, RTOL_ALPHA, f"pruned e_len L={L}")
+        assert np.all(a[keep == 0] == 0.0)
+
+
+def test_pruned_keep_all_is_unpruned():
+    """keep = L everywhere gives hs_feedback_topl's alphas bit for bit."""
+    w = W["llama3_batch"]
+    d = synth.make_inputs(w, device=DEV, seed=811, B=2, N=4, P=3)
+    keep = np.full(d["drafter"].shape[:3], 10, np.int32)
+    for greedy in (False, True):
+        a, e, st = run_pruned(d, w.temperature, greedy, 10, keep)
+        a0, e0, st0 = run(d, w.temperature, greedy, 10)
+        assert st == st0 == hf.HS_OK
+        assert np.array_equal(a, a0) and np.array_equal(e, e0)
+
+
+def test_pruned_keep_out_of_range():
+    """A kept count outside [0, L] makes only that alpha NaN and reports
+    HS_ERR_INVALID_ARG; a null keep pointer is refused before any launch."""
+    w = W["qwen3_8b_chain"]
+    d = synth.make_inputs(w, device=DEV, seed=812, B=2, N=2, P=3, V=5000)
+    keep = np.full((2, 2, 3), 2, np.int32)
+    keep[1, 0, 2] = 5
+    keep[0, 1, 1] = -1
+    a, e, st = run_pruned(d, 0.7, False, 4, keep)
+    assert st == hf.HS_ERR_INVALID_ARG
+    assert np.isnan(a[1, 0, 2]) and np.isnan(a[0, 1, 1]) and np.isnan(a).sum() == 2
+    ra, re, rst = oracle_pruned(d, 0.7, False, 4, keep)
+    assert rst == oracle.BADARG
+    assert_rel(a, ra, RTOL_ALPHA, "alpha next to a bad keep")
+    alpha = torch.empty(2, 2, 3, device=DEV)
+    st = hf.lib().hs_feedback_topl_pruned(
+        hf._ptr(d["target"]), hf._ptr(d["drafter"]), hf.HS_BF16, 2, 2, 3, 5000, 0.7, 0, 4, None,
+        hf._ptr(alpha), None, None, 0, None, None)
+    assert st == hf.HS_ERR_INVALID_ARG
