@@ -30,6 +30,7 @@ the data path); value = all ranks' evaluations / the slowest rank's time.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -67,6 +68,9 @@ def parse_args():
                          "the clock sampler")
     ap.add_argument("--cpu-budget-s", type=float, default=8.0,
                     help="seconds of oracle work per CPU-baseline leg (1 thread, all cores)")
+    ap.add_argument("--queries", type=int, default=0,
+                    help="run the workload with this many queries B instead of its own (a "
+                         "smaller case of the same kernels, for profiling)")
     ap.add_argument("--session", action="store_true",
                     help="long-session learner run: cumulative regret over the workload's rounds")
     ap.add_argument("--rounds", type=int, default=0, help="session rounds (0: the workload's)")
@@ -306,6 +310,8 @@ def run_ours(args):
     hf.lib()
 
     w = synth.WORKLOADS[args.workload]
+    if args.queries:
+        w = dataclasses.replace(w, B=args.queries, name=f"{w.name}_B{args.queries}")
     greedy = args.mode == "greedy"
     topl = args.mode == "topl"
     token = args.mode == "token"

@@ -36,7 +36,7 @@ namespace {
 constexpr int kConsumerWarps = 16;
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;       // + the producer warp
-constexpr int kStages = 6;                      // ring stages
+constexpr int kStages = 7;                      // ring stages (224 KB)
 constexpr int kVecsPerThread = 4;               // 16-byte vectors of a stage per consumer
 constexpr int kChunkVecs = kVecsPerThread * kConsumers;
 constexpr int kChunkBytes = kChunkVecs * 16;    // 32 KB
@@ -414,8 +414,9 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       for (int u = 0; u < kVecsPerThread; ++u)
         if (ch * kChunkVecs + u * kConsumers + t >= nvec) v[u] = make_uint4(ninf, ninf, ninf, ninf);
     }
-    __syncwarp();  // the warp's reads of the stage are done: hand it back
-    if (l == 0) mbar_arrive(saddr(&sh.empty[stage]));
+    // every consumer thread releases its own part of the stage (the stage's
+    // barrier counts kConsumers arrivals): no warp-level hand-off needed
+    mbar_arrive(saddr(&sh.empty[stage]));
     if (++stage == kStages) {
       stage = 0;
       phase ^= 1u;
@@ -575,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(saddr(&sh.full[s]), 1);
-      mbar_init(saddr(&sh.empty[s]), kConsumerWarps);
+      mbar_init(saddr(&sh.empty[s]), kConsumers);
     }
     sh.error = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
