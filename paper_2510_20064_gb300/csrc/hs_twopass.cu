@@ -154,6 +154,24 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint4 (&v)[4]) {
                   "r"(v[1].y), "r"(v[1].z), "r"(v[1].w), "r"(v[2].x), "r"(v[2].y), "r"(v[2].z),
                   "r"(v[2].w), "r"(v[3].x), "r"(v[3].y), "r"(v[3].z), "r"(v[3].w) : "memory");
 }
+// The load alone; tmem_wait_ld() below makes the registers valid.
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint4 (&v)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, "
+               "%9, %10, %11, %12, %13, %14, %15}, [%16];"
+               : "=r"(v[0].x), "=r"(v[0].y), "=r"(v[0].z), "=r"(v[0].w), "=r"(v[1].x),
+                 "=r"(v[1].y), "=r"(v[1].z), "=r"(v[1].w), "=r"(v[2].x), "=r"(v[2].y),
+                 "=r"(v[2].z), "=r"(v[2].w), "=r"(v[3].x), "=r"(v[3].y), "=r"(v[3].z),
+                 "=r"(v[3].w) : "r"(taddr) : "memory");
+}
+// Waits for this thread's tensor-memory loads; the registers are passed
+// through so that no use of them moves above the wait.
+__device__ __forceinline__ void tmem_wait_ld(uint4 (&v)[4]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(v[0].x), "+r"(v[0].y), "+r"(v[0].z), "+r"(v[0].w), "+r"(v[1].x),
+                 "+r"(v[1].y), "+r"(v[1].z), "+r"(v[1].w), "+r"(v[2].x), "+r"(v[2].y),
+                 "+r"(v[2].z), "+r"(v[2].w), "+r"(v[3].x), "+r"(v[3].y), "+r"(v[3].z),
+                 "+r"(v[3].w) :: "memory");
+}
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint4 (&v)[4]) {
   asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, "
                "%9, %10, %11, %12, %13, %14, %15}, [%16];"
@@ -332,13 +350,12 @@ __device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerTh
 }
 
 // Every lane: the merge (R, S) of the warp's pairs (R, s), each s relative to
-// its integer reference R: the largest reference first, then every sum
-// rescaled to it once (by an exact power of 2) and added up.  (R is never
-// NaN; a +inf R only comes with the row's bad flag.)
+// its integer reference R: the largest reference first (one redux), then
+// every sum rescaled to it once (by an exact power of 2) and added up.  (R is
+// never NaN; a +inf R only comes with the row's bad flag.)
 __device__ __forceinline__ void warp_merge(float& R, float& s) {
-  float M = R;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float M;
+  asm("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(M) : "f"(R));
   s = (R == -INFINITY) ? 0.f : s * ex2(R - M);
   R = M;
 #pragma unroll
@@ -484,11 +501,17 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     // drafters; sp: the split form (callers pass constants where they can, so
     // the loops below carry none of these tests)
     auto p2chunk = [&](int ch, bool tail, bool tm, bool full, bool sp) {
-      uint4 v[kVecsPerThread];
-      if (tm)
-        tmem_ld16(tcol + uint32_t(kWords * ch), v);
-      else
+      uint4 v[kVecsPerThread], d[kVecsPerThread];
+      // the target's words (tensor memory or ring) and the first drafter's:
+      // the tensor-memory load is in flight while the drafter's chunk is taken
+      if (tm) {
+        tmem_ld16_async(tcol + uint32_t(kWords * ch), v);
+        take(ch, tail, d);
+        tmem_wait_ld(v);
+      } else {
         take(ch, tail, v);
+        take(ch, tail, d);
+      }
       float xt[8 * kVecsPerThread];  // log2 p of the thread's 32 logits
 #pragma unroll
       for (int u = 0; u < kVecsPerThread; ++u) {
@@ -503,10 +526,10 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
 #pragma unroll
       for (int gi = 0; gi < kG; ++gi) {
         if (full || gi < g.dn) {
-          take(ch, tail, v);
+          if (gi > 0) take(ch, tail, d);
 #pragma unroll
           for (int u = 0; u < kVecsPerThread; ++u) {
-            const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+            const uint32_t wd[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               uint64_t e = fma2(pair_of<DT>(wd[q]), c2, od2[gi]);
