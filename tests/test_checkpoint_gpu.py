@@ -40,6 +40,9 @@ def e_len_of(a):
     return 1.0 + prod.sum(dim=-1)
 
 
+STREAM_FIELDS = ("gamma", "who", "n_tok", "n_done")  # the token stream's device arrays
+
+
 def fresh(kind):
     st = {"state": torch.zeros(N, B, device=DEV),
           "weights": torch.full((N, B), 1.0 / N, device=DEV),
@@ -47,26 +50,36 @@ def fresh(kind):
           "played": torch.zeros(B, device=DEV)}
     if kind == "token":
         ts = hf.TokenStream(N, B, K + 2 * P, DEV)
-        st.update(gamma=ts.gamma, who=ts.who, n_tok=ts.n_tok, n_done=ts.n_done)
+        st.update({f: getattr(ts, f) for f in STREAM_FIELDS})
     return st
 
 
+def stream_of(st):
+    """A TokenStream over the arrays in st (a fresh one, or one read back
+    from a checkpoint)."""
+    ts = hf.TokenStream(N, B, st["gamma"].shape[1], DEV)
+    for f in STREAM_FIELDS:
+        getattr(ts, f).copy_(st[f])
+    return ts
+
+
 def play(kind, learner, st, t0, t1, status):
+    ts = stream_of(st) if kind == "token" else None
     for t in range(t0, t1):
         a, k_h, u = round_inputs(t)
         if kind == "chunk":
             hf.hs_learner_step(a, e_len_of(a), hf.HS_LOSS_LENGTH, learner, ETA, st["state"],
                                st["weights"], st["sel"], played_loss=st["played"])
         else:
-            ts = hf.TokenStream.__new__(hf.TokenStream)
-            ts.N, ts.B, ts.H = N, B, st["gamma"].shape[1]
-            ts.gamma, ts.who, ts.n_tok, ts.n_done = st["gamma"], st["who"], st["n_tok"], st["n_done"]
             hf.hs_token_append(ts, a, k_h, st["sel"], dev_status=status)
             arg = torch.empty(B, dtype=torch.int32, device=DEV)
             hf.hs_token_learner_step(ts, K, hf.HS_LOSS_LENGTH, learner, ETA, st["state"],
                                      st["weights"], arg, played_loss=st["played"],
                                      dev_status=status)
             hf.hs_sample_select(st["weights"], u, selected=st["sel"], dev_status=status)
+    if ts is not None:  # the stream's arrays back into st
+        for f in STREAM_FIELDS:
+            st[f].copy_(getattr(ts, f))
 
 
 @pytest.mark.parametrize("kind", ["chunk", "token"])
