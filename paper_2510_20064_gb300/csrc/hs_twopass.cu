@@ -355,7 +355,7 @@ __device__ __forceinline__ void stat_chunk(Stat& st, const uint4 (&v)[kVecsPerTh
 // never NaN; a +inf R only comes with the row's bad flag.)
 __device__ __forceinline__ void warp_merge(float& R, float& s) {
   float M;
-  asm("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(M) : "f"(R));
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(M) : "f"(R));  // warp-collective: kept in place
   s = (R == -INFINITY) ? 0.f : s * ex2(R - M);
   R = M;
 #pragma unroll
