@@ -452,20 +452,28 @@ def run_ours(args):
     h2d = sum(v.numel() * v.element_size() for k, v in host_sets[0].items() if k != "sigma")
     d2h = out_w.numel() * 4 + out_s.numel() * 4
     e2e_steps = max(1, min(args.steps, args.e2e_steps))
+
+    def e2e_step(s):
+        hs = host_sets[s % 2]
+        for k, v in hs.items():
+            if k != "sigma":
+                dsts[k].copy_(v, non_blocking=True)
+        step(dsts)
+        out_w.copy_(weights, non_blocking=True)
+        out_s.copy_(sel, non_blocking=True)
+
     with torch.cuda.stream(stream):
+        # warm-up over both host sets: the first copy out of a freshly pinned
+        # buffer pays a one-time mapping cost of tens of milliseconds
+        for s in range(2 * max(1, math.ceil(args.warmup / 2))):
+            e2e_step(s)
         hdist.barrier(world, dev)
         torch.cuda.synchronize(dev)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for s in range(e2e_steps):
-            hs = host_sets[s % 2]
-            for k, v in hs.items():
-                if k != "sigma":
-                    dsts[k].copy_(v, non_blocking=True)
-            step(dsts)
-            out_w.copy_(weights, non_blocking=True)
-            out_s.copy_(sel, non_blocking=True)
+            e2e_step(s)
         e1.record(stream)
         torch.cuda.synchronize(dev)
     t_e2e = e0.elapsed_time(e1) / 1e3

@@ -257,3 +257,31 @@ def test_pruned_keep_out_of_range():
         hf._ptr(d["target"]), hf._ptr(d["drafter"]), hf.HS_BF16, 2, 2, 3, 5000, 0.7, 0, 4, None,
         hf._ptr(alpha), None, None, 0, None, None)
     assert st == hf.HS_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
+def test_pruned_dtypes_masks_and_extremes(dtype):
+    """Pruned candidate sets on every storage dtype, a ragged vocabulary with
+    masked (-inf) tokens, and the extreme counts: every child pruned (alpha
+    exactly 0) and none pruned, in one call."""
+    w = synth.Workload("pruned", N=3, B=2, P=4, V=20001, dtype=dtype, temperature=0.8,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=820)
+    mask = torch.rand(w.V, device=DEV) < 0.2
+    d["drafter"][..., mask] = float("-inf")
+    d["target"][..., mask.roll(3)] = float("-inf")
+    L = 7
+    rng = np.random.default_rng(821)
+    keep = rng.integers(0, L + 1, (w.N, w.B, w.P)).astype(np.int32)
+    keep[0] = 0
+    keep[1] = L
+    for greedy in (False, True):
+        a, e, st = run_pruned(d, w.temperature, greedy, L, keep)
+        ra, re, rst = oracle_pruned(d, w.temperature, greedy, L, keep)
+        assert st == hf.HS_OK and rst == 0, (st, rst)
+        if greedy:
+            assert np.array_equal(a, ra) and np.array_equal(e, re)
+        else:
+            assert_rel(a, ra, RTOL_ALPHA, f"pruned alpha {dtype}")
+            assert_rel(e, re, RTOL_ALPHA, f"pruned e_len {dtype}")
+        assert np.all(a[0] == 0.0) and np.all(e[0] == 1.0)
