@@ -210,26 +210,60 @@ struct Params {
   float c;
 };
 
-// A CTA's group: drafters d0 .. d0+dn-1 of one tile, starting at row index
-// r = tile * N + d0 of the run [r, re); up to kG drafters, ending at the
-// tile's last drafter or the run's end.
-// with_t: the group starts a tile or the run, so its pass 1 reads the target.
+// A CTA's group: drafters d0 .. d0+dn-1 of one tile, up to kG of them.
+// with_t: the group starts the run's segment of its tile, so its pass 1
+// reads the target; t_last: the segment's last group; shared: the tile has
+// drafters in a neighbouring run too.
 struct Group {
   int tile, d0, dn;
-  bool with_t, t_last;  // t_last: the tile's last group in this run
+  bool with_t, t_last, shared;
 };
-__device__ __forceinline__ Group group_at(int r, bool first, int re, int N) {
-  Group g;
-  g.tile = r / N;
-  g.d0 = r - g.tile * N;
-  int dn = kG;
-  if (dn > N - g.d0) dn = N - g.d0;
-  if (dn > re - r) dn = re - r;
-  g.dn = dn;
-  g.with_t = first || g.d0 == 0;
-  g.t_last = g.d0 + dn == N || r + dn == re;
-  return g;
-}
+
+// A CTA's walk over its run of drafter rows [rb, re) (tile-major), segment by
+// segment -- a segment is the part of the run in one tile -- and in groups of
+// up to kG drafters within a segment.  Even CTAs take the segments from the
+// run's last tile back to its first, odd CTAs from the first on, so a tile
+// split between two neighbouring runs is the first segment of both (read at
+// the start of the call) or the last segment of both (read in both CTAs'
+// final stretch): the second read of its target row can then come from L2.
+struct Walk {
+  int rb, re, N, tfirst, tlast, seg, tile, lo, hi, r;
+  bool rev;
+  __device__ void init(int rb_, int re_, int N_, bool rev_) {
+    rb = rb_;
+    re = re_;
+    N = N_;
+    rev = rev_;
+    tfirst = rb / N;
+    tlast = re > rb ? (re - 1) / N : tfirst - 1;
+    seg = 0;
+    if (!done()) start();
+  }
+  __device__ bool done() const { return seg > tlast - tfirst; }
+  __device__ void start() {
+    tile = rev ? tlast - seg : tfirst + seg;
+    lo = rb > tile * N ? rb : tile * N;
+    hi = re < (tile + 1) * N ? re : (tile + 1) * N;
+    r = lo;
+  }
+  __device__ Group group() const {
+    Group g;
+    g.tile = tile;
+    g.d0 = r - tile * N;
+    g.dn = hi - r < kG ? hi - r : kG;
+    g.with_t = r == lo;
+    g.t_last = r + g.dn == hi;
+    g.shared = lo > tile * N || hi < (tile + 1) * N;
+    return g;
+  }
+  __device__ void advance(int dn) {
+    r += dn;
+    if (r >= hi) {
+      ++seg;
+      if (!done()) start();
+    }
+  }
+};
 
 // ---- consumer warps ---------------------------------------------------------------
 
@@ -461,9 +495,10 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
   };
   Norm nt = {0.f, 0.f};   // normaliser of the current tile's target row
   bool bad_path = false;  // the current tile has an out-of-range path node
-  bool first = true;
-  for (int r = rb; r < re;) {
-    const Group g = group_at(r, first, re, p.N);
+  Walk walk;
+  walk.init(rb, re, p.N, (blockIdx.x & 1u) == 0u);
+  for (; !walk.done(); ) {
+    const Group g = walk.group();
     if (g.with_t) {
       bad_path = false;
       (void)target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path);
@@ -576,8 +611,7 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       }
     }
     rp ^= 1u;
-    r += g.dn;
-    first = false;
+    walk.advance(g.dn);
   }
   // every consumer warp is done with tensor memory before it is released
   tmem_fence_before();
@@ -646,9 +680,10 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
       auto drow = [&](int d, int tile) {
         return static_cast<const char*>(row_ptr<DT>(p.drafter, int64_t(d) * T + tile, p.V));
       };
-      bool first_group = true;
-      for (int r = rb; r < re;) {
-        const Group g = group_at(r, first_group, re, p.N);
+      Walk walk;
+      walk.init(rb, re, p.N, (blockIdx.x & 1u) == 0u);
+      for (; !walk.done(); ) {
+        const Group g = walk.group();
         bool bad_path = false;
         const char* tr = static_cast<const char*>(
             target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path));
@@ -662,8 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1) twopass_kernel(const Params p) {
           if (ch >= kTmemChunks) put(tr, ch, g.t_last ? once : keep);
           for (int gi = 0; gi < g.dn; ++gi) put(drow(g.d0 + gi, g.tile), ch, once);
         }
-        r += g.dn;
-        first_group = false;
+        walk.advance(g.dn);
       }
       if (!ok) {
         // the copies already issued must land before the CTA's memory goes
