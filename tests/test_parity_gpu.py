@@ -279,6 +279,62 @@ def test_streaming_kernel_many_tiles():
                "streaming e_len")
 
 
+def test_streaming_kernel_lagged_steps():
+    """Rows of 2 600 000 logits: 159 chunks per row, more than there are SMs,
+    so a tile's items span steps and each overlap comes two steps after its
+    statistics; every alpha and e_len is compared."""
+    w = synth.Workload("huge_vocab", N=2, B=1, P=2, V=2_600_000, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=23)
+    compare_full(d, 0.9, False)
+
+
+@pytest.mark.parametrize("T", [0.05, 5.0])
+def test_streaming_kernel_fp16_max_drafters(T):
+    """fp16, N = 32 (the most the kernel takes) and V = 160 000 at extreme
+    temperatures, with the first 100 000 logits of one query's rows masked to
+    -inf (its chunks' references come from the rest); every alpha and e_len
+    is compared.  At T = 0.05 the noisiest drafters barely overlap the target
+    (alpha ~1e-43), so alpha also gets the V * 2^-126 absolute floor of the
+    flush to zero below fp32's normal range."""
+    w = synth.Workload("big_vocab", N=32, B=2, P=2, V=160000, dtype="fp16", temperature=T,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=24)
+    d["target"][1, :, :100000] = float("-inf")
+    d["drafter"][:, 1, :, :100000] = float("-inf")
+    a, e, st = run(d, T, False)
+    ra, re, rst = oracle_feedback(d, T, False)
+    assert st == hf.HS_OK and rst == 0
+    assert_rel(a, ra, RTOL_ALPHA, "alpha", atol=w.V * 2.0 ** -126)
+    assert_rel(e, re, RTOL_ALPHA, "e_len")
+    assert np.nanmax(ra) > 0.1, "some pairs must overlap well above the flush floor"
+
+
+def test_streaming_kernel_flags_bad_rows():
+    """V above the cluster kernel's range: a NaN drafter logit in a row's last
+    chunk and a +inf one in its first only make their own alphas NaN
+    (HS_ERR_NONFINITE); an out-of-range path node makes its tile's alphas NaN
+    (HS_ERR_INVALID_ARG)."""
+    w = synth.Workload("big_vocab", N=3, B=4, P=3, V=200000, dtype="bf16", temperature=1.0,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=25)
+    d["drafter"][2, 3, 1, 199999] = float("nan")
+    d["drafter"][0, 1, 0, 7] = float("inf")
+    a, e, st = run(d, 1.0, False)
+    ra, re, rst = oracle_feedback(d, 1.0, False)
+    assert st == hf.HS_ERR_NONFINITE
+    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 2
+    assert np.isnan(a[2, 3, 1]) and np.isnan(a[0, 1, 0])
+    assert_rel(a, ra, RTOL_ALPHA, "alpha next to a NaN row")
+    t = synth.make_inputs(W["tree_path"], device=DEV, B=3, N=2, V=200000, seed=26)
+    t["path"][2, 1] = -1
+    a, e, st = run(t, 1.0, False)
+    assert st == hf.HS_ERR_INVALID_ARG
+    assert np.isnan(a[:, 2, 1]).all() and np.isnan(a).sum() == 2
+    t["path"][2, 1] = 3
+    compare_full(t, 1.0, False)
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "fp16"])
 def test_two_pass_kernel_every_alpha(dtype):
     """320 tiles of 76808-logit rows: the cluster kernel would hold them on 144
