@@ -405,9 +405,9 @@ hs_status hs_schedule_next(const hs_schedule_config* cfg, hs_schedule_state* sta
  * Exercises the bounded-wait error path of the library's kernels on a GPU
  * without faulting or hanging it.  It runs the streaming stochastic kernel
  * (the one hs_feedback uses for V > 153 600) with one change: the wait of
- * tile (b,k) = (0,0) for its statistics asks for one chunk more than exist,
- * so it can only run out, and every wait is limited to `wait_cycles` SM clock
- * cycles instead of about a second.  Tile (0,0)'s waits then report
+ * tile (b,k) = (0,0) for its statistics asks for one count more than exist,
+ * so it can only run out, and every wait on a tile's statistics count is
+ * limited to `wait_cycles` SM clock cycles instead of about a second.  Tile (0,0)'s waits then report
  * HS_ERR_TIMEOUT to *dev_status and its alphas (and the e_len of query 0)
  * come out NaN; every other alpha is the one hs_feedback computes, and the
  * CUDA context stays usable.  Same arguments as hs_feedback (stochastic,
