@@ -312,19 +312,20 @@ def test_streaming_kernel_fp16_max_drafters(T):
 
 def test_streaming_kernel_flags_bad_rows():
     """V above the cluster kernel's range: a NaN drafter logit in a row's last
-    chunk and a +inf one in its first only make their own alphas NaN
-    (HS_ERR_NONFINITE); an out-of-range path node makes its tile's alphas NaN
-    (HS_ERR_INVALID_ARG)."""
+    chunk, a +inf one in its first and a drafter row with no finite logit only
+    make their own alphas NaN (HS_ERR_NONFINITE); an out-of-range path node
+    makes its tile's alphas NaN (HS_ERR_INVALID_ARG)."""
     w = synth.Workload("big_vocab", N=3, B=4, P=3, V=200000, dtype="bf16", temperature=1.0,
                        target="zipf", sigma="qwen")
     d = synth.make_inputs(w, device=DEV, seed=25)
     d["drafter"][2, 3, 1, 199999] = float("nan")
     d["drafter"][0, 1, 0, 7] = float("inf")
+    d["drafter"][1, 2, 2, :] = float("-inf")
     a, e, st = run(d, 1.0, False)
     ra, re, rst = oracle_feedback(d, 1.0, False)
     assert st == hf.HS_ERR_NONFINITE
-    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 2
-    assert np.isnan(a[2, 3, 1]) and np.isnan(a[0, 1, 0])
+    assert np.array_equal(np.isnan(a), np.isnan(ra)) and np.isnan(a).sum() == 3
+    assert np.isnan(a[2, 3, 1]) and np.isnan(a[0, 1, 0]) and np.isnan(a[1, 2, 2])
     assert_rel(a, ra, RTOL_ALPHA, "alpha next to a NaN row")
     t = synth.make_inputs(W["tree_path"], device=DEV, B=3, N=2, V=200000, seed=26)
     t["path"][2, 1] = -1
