@@ -5,11 +5,11 @@
 //                           max of the stored logits and the first index
 //                           holding it; every logit is read once, 8 16-byte
 //                           loads in flight per thread
-//   greedy_finalize_kernel  one warp per drafter row (i, b, k): combines the
-//                           chunk partials of its target and drafter rows in
-//                           chunk order (first index wins ties) and compares;
-//                           the last of the P warps of (i, b) to finish (an
-//                           atomic count the argmax kernel zeroes) forms e_len
+//   greedy_finalize_kernel  one warp per (drafter i, query b), lane k for
+//                           position k: combines the chunk partials of its
+//                           target and drafter rows in chunk order (first
+//                           index wins ties) and compares; the warp's prefix
+//                           products of alpha then give e_len (no atomics)
 // All of it is exact: maxima and indices of the stored values.
 #include <math.h>
 #include <stdint.h>
@@ -36,10 +36,8 @@ template <int DT, bool VEC>
 __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
     const void* __restrict__ target, const int32_t* __restrict__ path, int M,
     const void* __restrict__ drafter, int B, int P, int V, Part* __restrict__ parts,
-    int nchunk, int* __restrict__ counters, int ncounters) {
+    int nchunk) {
   pdl_wait();
-  if (counters && blockIdx.x == 0 && blockIdx.y == 0)
-    for (int x = threadIdx.x; x < ncounters; x += kThreads) counters[x] = 0;
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kS = kUnroll * kV;
   __shared__ float red_m[kWarps];
@@ -84,68 +82,67 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
   pdl_trigger();
 }
 
-// Row argmax from its chunk partials, by one warp: (max, first index).
+// Row argmax from its chunk partials, by one thread, chunks in order: the
+// strict '>' keeps the first chunk holding the max (each chunk's index is its
+// first); a NaN or +inf max makes the row unusable (checked by the caller).
 __device__ __forceinline__ void combine(const Part* __restrict__ pr, int nchunk, float& m,
                                         int& arg) {
-  const int l = threadIdx.x & 31;
-  float lm = -INFINITY;
-  int la = INT_MAX;
-  for (int j = l; j < nchunk; j += 32) {  // increasing chunk order per lane
+  m = -INFINITY;
+  arg = INT_MAX;
+  for (int j = 0; j < nchunk; ++j) {
     const Part q = pr[j];
-    if (q.m > lm || q.m != q.m) {
-      lm = q.m;
-      la = q.idx;
+    if (q.m > m || q.m != q.m) {
+      m = q.m;
+      arg = q.idx;
+      if (q.m != q.m) break;  // NaN: the row is unusable whatever follows
     }
   }
-  m = warp_max_nan(lm);
-  arg = warp_min_int(lm == m ? la : INT_MAX);
 }
 
 __global__ void greedy_finalize_kernel(const Part* __restrict__ parts, int nchunk,
                                        const int32_t* __restrict__ path, int M, int N, int B,
                                        int P, float* __restrict__ alpha,
-                                       float* __restrict__ e_len, int* __restrict__ counters,
-                                       int* dev_status) {
+                                       float* __restrict__ e_len, int* dev_status) {
   pdl_wait();
-  const int64_t r = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;  // row (i, b, k)
-  const int64_t BP = int64_t(B) * P;
-  if (r >= int64_t(N) * BP) return;  // whole warp
+  const int64_t ib = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;  // (i, b)
+  if (ib >= int64_t(N) * B) return;  // whole warp
   const int l = threadIdx.x & 31;
-  const int64_t tile = r % BP;
-  float mt, md;
-  int at, ad;
-  combine(parts + tile * nchunk, nchunk, mt, at);
-  combine(parts + (BP + r) * nchunk, nchunk, md, ad);
-  const bool bad_path = path && (path[tile] < 0 || path[tile] >= M);
-  int last = 0;
-  if (l == 0) {
-    float a;
-    if (bad_path || !isfinite(mt) || !isfinite(md)) {
-      a = __int_as_float(0x7fc00000);
-      report(dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
-    } else {
-      a = (at == ad) ? 1.f : 0.f;
+  const int64_t BP = int64_t(B) * P, i = ib / B, b = ib - i * B;
+  // e_len = 1 + sum_{k < P-1} prod_{j <= k} alpha_j, 32 positions at a time:
+  // an inclusive prefix product over the lanes, carried between groups
+  float e = 1.f, carry = 1.f;
+  for (int k0 = 0; k0 < P; k0 += 32) {
+    const int k = k0 + l;
+    float a = 1.f;
+    if (k < P) {
+      const int64_t tile = b * P + k;
+      float mt, md;
+      int at, ad;
+      combine(parts + tile * nchunk, nchunk, mt, at);
+      combine(parts + (BP + i * BP + tile) * nchunk, nchunk, md, ad);
+      const bool bad_path = path && (path[tile] < 0 || path[tile] >= M);
+      if (bad_path || !isfinite(mt) || !isfinite(md)) {
+        a = __int_as_float(0x7fc00000);
+        report(dev_status, bad_path ? HS_ERR_INVALID_ARG : HS_ERR_NONFINITE);
+      } else {
+        a = (at == ad) ? 1.f : 0.f;
+      }
+      alpha[ib * P + k] = a;
     }
-    alpha[r] = a;
-    if (e_len) {
-      __threadfence();  // alpha[r] before the count
-      last = atomicAdd(&counters[r / P], 1) == P - 1;
+    float pp = k < P - 1 ? a : 1.f;  // positions from P-1 on enter no product
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float up = __shfl_up_sync(0xffffffffu, pp, o);
+      if (l >= o) pp *= up;
     }
+    const float term = k < P - 1 ? carry * pp : 0.f;
+    e += warp_sum(term);
+    carry *= __shfl_sync(0xffffffffu, pp, 31);
   }
-  // the last warp of (i, b) forms e_len = 1 + sum_{k<K} prod_{j<=k} alpha_j
-  if (__shfl_sync(0xffffffffu, last, 0) && l == 0) {
-    __threadfence();
-    const int64_t ib = r / P;
-    float e = 1.f, prod = 1.f;
-    for (int k = 0; k < P - 1; ++k) {
-      prod *= __ldcg(alpha + ib * P + k);
-      e += prod;
-    }
-    e_len[ib] = e;
-  }
+  if (e_len && l == 0) e_len[ib] = e;
 }
 
-// Partials, then one counter per (i, b) at the next 256-byte boundary.
+// One partial per (row, chunk).
 size_t parts_bytes(int N, int B, int P, int V, int dtype) {
   const int64_t ch = dtype == HS_FP32 ? chunk_of<HS_FP32>() : chunk_of<HS_BF16>();
   const int64_t nchunk = (V + ch - 1) / ch;
@@ -160,17 +157,12 @@ hs_status launch_t(const void* target, const int32_t* path, int M, const void* d
   Part* parts = static_cast<Part*>(ws);
   const int nchunk = int((V + chunk_of<DT>() - 1) / chunk_of<DT>());
   const unsigned rows = unsigned(int64_t(B) * P * (int64_t(N) + 1));
-  int* counters = e_len ? reinterpret_cast<int*>(static_cast<char*>(ws) +
-                                                  parts_bytes(N, B, P, V, DT))
-                        : nullptr;
   if (launch_pdl(argmax_chunk_kernel<DT, VEC>, dim3(rows, unsigned(nchunk)), dim3(kThreads), 0,
-                 s, target, path, M, drafter, B, P, V, parts, nchunk, counters,
-                 N * B) != cudaSuccess)
+                 s, target, path, M, drafter, B, P, V, parts, nchunk) != cudaSuccess)
     return HS_ERR_CUDA;
-  const int64_t threads = int64_t(N) * B * P * 32;
+  const int64_t threads = int64_t(N) * B * 32;
   if (launch_pdl(greedy_finalize_kernel, dim3(unsigned((threads + 255) / 256)), dim3(256), 0, s,
-                 parts, nchunk, path, M, N, B, P, alpha, e_len, counters,
-                 dev_status) != cudaSuccess)
+                 parts, nchunk, path, M, N, B, P, alpha, e_len, dev_status) != cudaSuccess)
     return HS_ERR_CUDA;
   return HS_OK;
 }
@@ -193,7 +185,7 @@ int64_t chunk_elems(int dtype) {
 }
 
 size_t workspace_bytes(int N, int B, int P, int V, int dtype) {
-  return parts_bytes(N, B, P, V, dtype) + size_t(N) * B * sizeof(int);
+  return parts_bytes(N, B, P, V, dtype);
 }
 
 hs_status launch(bool vec, const void* target, const int32_t* path, int M, const void* drafter,

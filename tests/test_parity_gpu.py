@@ -241,6 +241,21 @@ def test_drafter_counts(N):
     compare_full(d, 1.0, False)
 
 
+@pytest.mark.parametrize("greedy", [False, True])
+def test_long_chain(greedy):
+    """P = 40 scored positions (more than a warp's 32 lanes): the greedy
+    finalize carries its prefix product of alpha from one group of 32
+    positions to the next; drafter 0 copies the target, so its alphas are 1
+    at every position and e_len reaches P.  Every alpha and e_len compared."""
+    w = synth.Workload("long_chain", N=3, B=2, P=40, V=4096, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=12)
+    d["drafter"][0] = d["target"]
+    a, e = compare_full(d, 0.9, greedy)
+    if greedy:
+        assert np.all(a[0] == 1.0) and np.all(e[0] == 40.0)
+
+
 def test_more_tiles_than_resident_clusters():
     """B*P = 1200 tiles: every resident cluster loops over many tiles."""
     w = W["qwen3_8b_chain"]
