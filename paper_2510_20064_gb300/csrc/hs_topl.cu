@@ -36,7 +36,11 @@ namespace hs {
 namespace topl {
 namespace {
 
-constexpr int kThreads = 256;
+// Small CTAs (4 independent warps): the SMs then get nearly equal shares of
+// the warps (tree_path's 2048 rows are 512 CTAs, 3 or 4 per SM, where 256
+// CTAs of 8 warps gave some SMs twice the work of others), and the register
+// budget of 4 CTAs per SM (128) holds the warp's state without spilling.
+constexpr int kThreads = 128;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;                        // 16-byte vectors per lane per step
 constexpr int kStages = 3;                        // ring stages per warp
@@ -637,7 +641,7 @@ __global__ void __launch_bounds__(kThreads) alpha_kernel(const Params p) {
 // Warps per row: enough that the GPU holds about kWarpTarget warps when rows
 // are few (at most 16, and never more parts than whole steps in the row).
 constexpr int64_t kFewRows = 1216;     // below this many rows a row is split
-constexpr int64_t kWarpTarget = 4864;  // 152 SMs x 32 warps: one full wave of topl_kernel
+constexpr int64_t kWarpTarget = 4864;  // 152 SMs x 32 warps
 int split_of(int64_t rows, int V) {
   if (rows > kFewRows) return 1;  // splitting adds insertions; only for few rows
   int64_t S = (kWarpTarget + rows - 1) / rows;
