@@ -955,8 +955,12 @@ hs_status launch(const void* target, const int32_t* path, int M, const void* dra
   const int cluster_sms =
       pl.C * (dtype == HS_BF16 ? clusters_of<HS_BF16>(pl) : clusters_of<HS_FP16>(pl));
   hs_status st;
+  const int pairs = twopass::pair_grid(V, 2, B * P, N, sms, size_t(l2));
   if (twopass::preferred(V, 2, B * P, N, sms, cluster_sms, size_t(l2)))
     st = twopass::launch(target, path, M, drafter, dtype, N, B, P, V, c, 0, sms, alpha,
+                         dev_status, stream);
+  else if (pairs > 0)  // one CTA per drafter pair
+    st = twopass::launch(target, path, M, drafter, dtype, N, B, P, V, c, 0, pairs, alpha,
                          dev_status, stream);
   else
     st = dtype == HS_BF16 ? launch_dt<HS_BF16>(p, pl, stream) : launch_dt<HS_FP16>(p, pl, stream);

@@ -726,6 +726,16 @@ bool preferred(int V, int elem_bytes, int tiles, int N, int sms, int cluster_sms
   return working_set <= 0.9 * double(l2_bytes);
 }
 
+int pair_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes) {
+  const int64_t rows = int64_t(tiles) * N;
+  if (N % kG != 0 || rows >= 2 * int64_t(sms) || 10 * (rows / kG) < 7 * int64_t(sms)) return 0;
+  const int64_t grid = rows / kG;
+  const double row = double(V) * elem_bytes;
+  const double tail = row - double(kTmemChunks) * kChunkBytes;
+  const double working_set = (kG * row + (tail > 0 ? tail : 0.0)) * double(grid);
+  return working_set <= 0.9 * double(l2_bytes) ? int(grid) : 0;
+}
+
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
                  int N, int B, int P, int V, float c, int t0, int grid, float* alpha,
                  int* dev_status, cudaStream_t stream) {

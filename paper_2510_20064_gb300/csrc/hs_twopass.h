@@ -19,6 +19,13 @@ namespace twopass {
 bool preferred(int V, int elem_bytes, int tiles, int N, int sms, int cluster_sms,
                size_t l2_bytes);
 
+// The grid for calls with fewer than two drafter rows per SM whose drafters
+// pair up within tiles (N even): one CTA per pair of rows, when that keeps
+// at least 70% of the SMs busy and the pairs' working set fits in 90% of L2;
+// else 0.  (4 drafters x 56 tiles of 151 936 logits: 112 CTAs, 30.1 us per
+// call against the cluster kernel's 30.9.)
+int pair_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes);
+
 // alpha of tiles t0 .. B*P-1 (bf16/fp16, V % 8 == 0, 16-byte-aligned rows)
 // over `grid` CTAs (one per SM), each taking an even, contiguous run of the
 // drafter rows (tile-major).

@@ -384,6 +384,17 @@ def test_two_pass_kernel_flags_bad_rows():
     assert np.isnan(a[:, 79, 2]).all() and np.isnan(a).sum() == 2
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "fp16"])
+def test_two_pass_kernel_one_pair_per_cta(dtype):
+    """224 drafter rows (N = 4, 56 tiles): fewer than two per SM, so the
+    two-pass kernel runs one CTA per pair of drafters of a tile (112 CTAs),
+    each reading its tile's target row; every alpha and e_len is compared."""
+    w = synth.Workload("pairs", N=4, B=8, P=7, V=76808, dtype=dtype, temperature=0.7,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=49)
+    compare_full(d, 0.7, False)
+
+
 def test_two_pass_kernel_groups_cross_tiles():
     """N = 5 drafters: the 1600 drafter rows are split evenly over the SMs in
     runs that start and end inside tiles (such a run reads the tile's target
