@@ -187,13 +187,14 @@ __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" :: "n"(kConsumers) : "memory");
 }
 
-// Per-warp partials of one consumer barrier, double-buffered: buffer b is
-// rewritten two barriers later, after a barrier that every reader of its
-// previous contents has passed.
+// Per-warp posts of a group (the statistics of its rows, then its alpha
+// partials), double-buffered by group parity: a buffer is rewritten two
+// groups later, after barriers that every reader of its previous contents
+// has passed.
 struct Shared {
   uint64_t full[kStages], empty[kStages];
-  float m[2][kConsumerWarps], s[2][kConsumerWarps];
-  int bad[2][kConsumerWarps];
+  float m[2][1 + kG][kConsumerWarps], s[2][1 + kG][kConsumerWarps];  // [group parity][row]
+  int bad[2][1 + kG][kConsumerWarps];
   float acc[2][kG][kConsumerWarps];
   int error;
   uint32_t tmem_base;
@@ -473,10 +474,11 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
       phase ^= 1u;
     }
   };
-  uint32_t rp = 0;  // partial buffer of the next consumer barrier
-  // pass 1 over one row: its normaliser in every thread (NaN for an unusable
-  // row); park: the row's first kTmemChunks chunks also go to tensor memory
-  auto pass1 = [&](bool park) -> Norm {
+  uint32_t rp = 0;  // buffers of the current group (group parity)
+  // pass 1 over one row: each warp posts its merged statistics in slot
+  // `slot` of the group (0: the target, 1 + i: drafter i of the group);
+  // park: the row's first kTmemChunks chunks also go to tensor memory
+  auto pass1 = [&](bool park, int slot) {
     Stat st = stat_init<DT>();
     auto step = [&](int ch, bool tail) {
       uint4 v[kVecsPerThread];
@@ -487,11 +489,12 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
     for (int ch = 0; ch < nch - 1; ++ch) step(ch, false);
     step(nch - 1, true);
     if (park) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-    post_stat(st, sh.m[rp], sh.s[rp], sh.bad[rp], w, l);
-    consumer_sync();
-    const Norm n = row_norm(sh.m[rp], sh.s[rp], sh.bad[rp], l);
-    rp ^= 1u;
-    return n;
+    post_stat(st, sh.m[rp][slot], sh.s[rp][slot], sh.bad[rp][slot], w, l);
+  };
+  // after the group's consumer barrier: a row's normaliser in every thread
+  // (NaN for an unusable row)
+  auto norm_of = [&](int slot) {
+    return row_norm(sh.m[rp][slot], sh.s[rp][slot], sh.bad[rp][slot], l);
   };
   Norm nt = {0.f, 0.f};   // normaliser of the current tile's target row
   bool bad_path = false;  // the current tile has an out-of-range path node
@@ -499,14 +502,21 @@ __device__ __forceinline__ void consumer(const Params& p, Shared& sh, uint32_t r
   walk.init(rb, re, p.N, (blockIdx.x & 1u) == 0u);
   for (; !walk.done(); ) {
     const Group g = walk.group();
+    // pass 1 over the group's rows, each warp posting its statistics; one
+    // consumer barrier, then every warp merges the posts of each row
     if (g.with_t) {
       bad_path = false;
       (void)target_row<DT>(p.target, p.path, p.M, p.P, g.tile, p.V, &bad_path);
-      nt = pass1(true);
+      pass1(true, 0);
     }
+#pragma unroll
+    for (int gi = 0; gi < kG; ++gi)
+      if (gi < g.dn) pass1(false, 1 + gi);
+    consumer_sync();
+    if (g.with_t) nt = norm_of(0);
     Norm nd[kG];
 #pragma unroll
-    for (int gi = 0; gi < kG; ++gi) nd[gi] = gi < g.dn ? pass1(false) : Norm{0.f, 0.f};
+    for (int gi = 0; gi < kG; ++gi) nd[gi] = gi < g.dn ? norm_of(1 + gi) : Norm{0.f, 0.f};
     // The folded form takes each row's normaliser as one offset o = R + L,
     // held in fp32 to ulp(o)/2: alpha stays within 2.6e-6 relative while
     // |o| < kFoldLimit.  Otherwise (low temperatures, large logits) pass 2
