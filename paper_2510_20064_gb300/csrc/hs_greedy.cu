@@ -1,10 +1,10 @@
 // hs_greedy.cu -- greedy feedback: alpha = [argmax q_i == argmax p]
 // (Thm 2 with branching L = 1 under a greedy target), e_len by Thm 3.
 //
-//   argmax_chunk_kernel     one CTA per (row, 16K-logit chunk): NaN-propagating
+//   argmax_chunk_kernel     one CTA per (row, 32K-logit chunk): NaN-propagating
 //                           max of the stored logits and the first index
-//                           holding it; every logit is read once, 8 16-byte
-//                           loads in flight per thread
+//                           holding it; every logit is read once, each thread
+//                           issuing its 16 16-byte loads before using any
 //   greedy_finalize_kernel  one warp per (drafter i, query b), lane k for
 //                           position k: combines the chunk partials of its
 //                           target and drafter rows in chunk order (first
@@ -25,7 +25,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kUnroll = 8;
+constexpr int kUnroll = 16;
 
 template <int DT>
 __host__ __device__ constexpr int64_t chunk_of() {
@@ -50,7 +50,34 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
                            : row_ptr<DT>(drafter, r - BP, V);
   const int64_t v0 = int64_t(j) * chunk_of<DT>();
   float x[kS];
-  load_chunk<DT, VEC, kThreads, kUnroll>(row, v0, V, x);
+  if (VEC && DT != HS_FP32) {  // all 16 loads in flight first, then the widening
+    uint4 raw[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t v = v0 + int64_t(u * kThreads + threadIdx.x) * kV;
+      raw[u] = v < V ? __ldg(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(row) + v))
+                     : make_uint4(DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t wd[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (DT == HS_BF16) {
+          x[u * kV + 2 * q] = __uint_as_float(wd[q] << 16);
+          x[u * kV + 2 * q + 1] = __uint_as_float(wd[q] & 0xffff0000u);
+        } else {
+          x[u * kV + 2 * q] = __half2float(__ushort_as_half(static_cast<unsigned short>(wd[q] & 0xffffu)));
+          x[u * kV + 2 * q + 1] = __half2float(__ushort_as_half(static_cast<unsigned short>(wd[q] >> 16)));
+        }
+      }
+    }
+  } else {
+    load_chunk<DT, VEC, kThreads, kUnroll>(row, v0, V, x);
+  }
   // slots visit increasing v, so a strict '>' keeps the first index; a NaN
   // replaces m and then stays
   float m = -INFINITY;
