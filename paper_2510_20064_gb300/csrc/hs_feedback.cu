@@ -319,9 +319,16 @@ hs_status feedback_common(const void* target, const int32_t* path, int M, const 
   if (fused::eligible(target, drafter, dtype, N, V, greedy))
     return fused::launch(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, dev_status,
                          s);
-  if (stream::eligible(target, drafter, dtype, N, V, greedy))
+  if (stream::eligible(target, drafter, dtype, N, V, greedy)) {
+    // longer rows: the two-pass kernel while the rows are many enough and
+    // L2 still holds a good part of their second passes, else streaming
+    const int grid = fused::long_row_grid(N, B, P, V);
+    if (grid > 0)
+      return fused::launch_two_pass(target, path, M, drafter, dtype, N, B, P, V, c, grid, alpha,
+                                    e_len, dev_status, s);
     return stream::launch(target, path, M, drafter, dtype, N, B, P, V, c, alpha, e_len, ws,
                           dev_status, s);
+  }
   switch (dtype) {
     case HS_BF16:
       return dispatch_vec<HS_BF16>(vec, target, path, M, drafter, N, B, P, V, c, alpha, e_len,

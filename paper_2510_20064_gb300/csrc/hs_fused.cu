@@ -912,6 +912,30 @@ __global__ void elen_kernel(const float* __restrict__ alpha, int64_t NB, int P,
 
 }  // namespace
 
+int long_row_grid(int N, int B, int P, int V) {
+  int dev = 0, sms = 0, l2 = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
+    return 0;
+  return twopass::long_row_grid(V, 2, B * P, N, sms, size_t(l2));
+}
+
+hs_status launch_two_pass(const void* target, const int32_t* path, int M, const void* drafter,
+                          int dtype, int N, int B, int P, int V, float c, int grid, float* alpha,
+                          float* e_len, int* dev_status, cudaStream_t stream) {
+  const hs_status st = twopass::launch(target, path, M, drafter, dtype, N, B, P, V, c, 0, grid,
+                                       alpha, dev_status, stream);
+  if (st != HS_OK) return st;
+  if (e_len) {
+    const int64_t nb = int64_t(N) * B;
+    if (launch_pdl(elen_kernel, dim3(unsigned((nb + 255) / 256)), dim3(256), 0, stream, alpha,
+                   nb, P, e_len) != cudaSuccess)
+      return HS_ERR_CUDA;
+  }
+  return HS_OK;
+}
+
 bool eligible_sizes(int dtype, int N, int V, int greedy) {
   if (greedy || (dtype != HS_BF16 && dtype != HS_FP16)) return false;
   if (N > kMaxN || V % 8 != 0) return false;

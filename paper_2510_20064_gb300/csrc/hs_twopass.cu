@@ -746,6 +746,15 @@ int pair_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes)
   return working_set <= 0.9 * double(l2_bytes) ? int(grid) : 0;
 }
 
+int long_row_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes) {
+  const int64_t rows = int64_t(tiles) * N;
+  if (rows < 2 * int64_t(sms)) return pair_grid(V, elem_bytes, tiles, N, sms, l2_bytes);
+  const double row = double(V) * elem_bytes;
+  const double tail = row - double(kTmemChunks) * kChunkBytes;
+  const double working_set = (kG * row + (tail > 0 ? tail : 0.0)) * sms;
+  return working_set <= 2.0 * double(l2_bytes) ? sms : 0;
+}
+
 hs_status launch(const void* target, const int32_t* path, int M, const void* drafter, int dtype,
                  int N, int B, int P, int V, float c, int t0, int grid, float* alpha,
                  int* dev_status, cudaStream_t stream) {

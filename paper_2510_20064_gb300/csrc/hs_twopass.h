@@ -26,6 +26,14 @@ bool preferred(int V, int elem_bytes, int tiles, int N, int sms, int cluster_sms
 // call against the cluster kernel's 30.9.)
 int pair_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes);
 
+// The grid for rows longer than the cluster kernel holds (V > 153 600): one
+// CTA per SM when there are two drafter rows per SM or more and the SMs'
+// working sets (as for preferred()) come to at most twice L2 -- the second
+// passes then partly miss L2, but measured on V = 200 000 and 262 144 the call
+// still took 1.36-1.45x less time than the streaming kernel's -- else
+// pair_grid(); 0 leaves the call to the streaming kernel.
+int long_row_grid(int V, int elem_bytes, int tiles, int N, int sms, size_t l2_bytes);
+
 // alpha of tiles t0 .. B*P-1 (bf16/fp16, V % 8 == 0, 16-byte-aligned rows)
 // over `grid` CTAs (one per SM), each taking an even, contiguous run of the
 // drafter rows (tile-major).

@@ -278,20 +278,34 @@ def test_fp16_full_vocab():
 
 
 def test_streaming_kernel_many_tiles():
-    """V above the cluster kernel's range with many tiles per CTA."""
-    w = synth.Workload("big_vocab", N=5, B=24, P=4, V=200000, dtype="bf16", temperature=0.9,
+    """V above the cluster kernel's range with many tiles per CTA and 240
+    drafter rows of an odd N (fewer than two per SM, no drafter pairs), so the
+    streaming kernel takes the call."""
+    w = synth.Workload("big_vocab", N=5, B=24, P=2, V=200000, dtype="bf16", temperature=0.9,
                        target="zipf", sigma="qwen")
     d = synth.make_inputs(w, device=DEV, seed=21)
     a, e, st = run(d, 0.9, False)
     assert st == 0
     rng = np.random.default_rng(4)
-    samples = [(int(rng.integers(5)), int(rng.integers(24)), int(rng.integers(4)))
+    samples = [(int(rng.integers(5)), int(rng.integers(24)), int(rng.integers(2)))
                for _ in range(30)]
     ref = oracle_alpha_rows(d, samples, 0.9, False)
     assert_rel(np.array([a[s] for s in samples]), ref, RTOL_ALPHA, "streaming alpha")
-    col = oracle_alpha_rows(d, [(2, 7, k) for k in range(4)], 0.9, False)
+    col = oracle_alpha_rows(d, [(2, 7, k) for k in range(2)], 0.9, False)
     assert_rel(np.array([e[2, 7]]), np.array([1.0 + np.cumprod(col[:-1]).sum()]), RTOL_ALPHA,
                "streaming e_len")
+
+
+@pytest.mark.parametrize("N,B,P", [(2, 80, 2), (4, 8, 7)])
+def test_two_pass_kernel_long_rows(N, B, P):
+    """Rows of 200 000 logits, longer than the cluster kernel holds: with 320
+    drafter rows the two-pass kernel takes the call on every SM (its L2 working
+    set above L2, so some second passes come from HBM), with 224 rows of
+    N = 4 one CTA per drafter pair; every alpha and e_len is compared."""
+    w = synth.Workload("long_rows", N=N, B=B, P=P, V=200000, dtype="bf16", temperature=0.9,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=22 + N)
+    compare_full(d, 0.9, False)
 
 
 def test_streaming_kernel_lagged_steps():
