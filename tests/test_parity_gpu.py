@@ -409,6 +409,20 @@ def test_two_pass_kernel_one_pair_per_cta(dtype):
     compare_full(d, 0.7, False)
 
 
+@pytest.mark.parametrize("V,dtype", [(32776, "bf16"), (36872, "fp16"), (200000, "fp16")])
+def test_two_pass_kernel_short_last_chunk(V, dtype):
+    """Rows whose last 16 384-logit chunk is at most half full, where each
+    warp stops that chunk's arithmetic after its last vector holding logits:
+    one 8-logit vector in the last chunk (V = 32776, so warps 1-15 have none),
+    513 vectors (V = 36872, one lane of warp 0 holds a second vector), and
+    424 vectors (V = 200000, warps 14 and 15 have none).  One CTA per drafter
+    pair; every alpha and e_len is compared."""
+    w = synth.Workload("pairs", N=4, B=8, P=7, V=V, dtype=dtype, temperature=0.8,
+                       target="zipf", sigma="qwen")
+    d = synth.make_inputs(w, device=DEV, seed=53 + V)
+    compare_full(d, 0.8, False)
+
+
 def test_two_pass_kernel_groups_cross_tiles():
     """N = 5 drafters: the 1600 drafter rows are split evenly over the SMs in
     runs that start and end inside tiles (such a run reads the tile's target
