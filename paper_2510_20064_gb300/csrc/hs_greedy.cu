@@ -4,7 +4,9 @@
 //   argmax_chunk_kernel     one CTA per (row, 32K-logit chunk): NaN-propagating
 //                           max of the stored logits and the first index
 //                           holding it; every logit is read once, each thread
-//                           issuing its 16 16-byte loads before using any
+//                           issuing its 16 16-byte loads before using any;
+//                           only a row's ragged last chunk checks each slot
+//                           against V
 //   greedy_finalize_kernel  one warp per (drafter i, query b), lane k for
 //                           position k: combines the chunk partials of its
 //                           target and drafter rows in chunk order (first
@@ -32,34 +34,26 @@ __host__ __device__ constexpr int64_t chunk_of() {
   return int64_t(kThreads) * kUnroll * Elem<DT>::kVec;
 }
 
-template <int DT, bool VEC>
-__global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
-    const void* __restrict__ target, const int32_t* __restrict__ path, int M,
-    const void* __restrict__ drafter, int B, int P, int V, Part* __restrict__ parts,
-    int nchunk) {
-  pdl_wait();
+// This thread's max of one chunk of a row and the first index holding it
+// (INT_MAX when the chunk has no logit above -inf).  FULL: the chunk lies
+// inside the row, so no slot needs a bounds check.
+template <int DT, bool VEC, bool FULL>
+__device__ __forceinline__ void chunk_argmax(const void* row, int64_t v0, int V, float& m,
+                                             int& arg) {
   constexpr int kV = Elem<DT>::kVec;
   constexpr int kS = kUnroll * kV;
-  __shared__ float red_m[kWarps];
-  __shared__ int red_a[kWarps];
-  const int64_t r = blockIdx.x;
-  const int j = blockIdx.y;
-  const int64_t BP = int64_t(B) * P;
-  bool bad_path = false;
-  const void* row = r < BP ? target_row<DT>(target, path, M, P, r, V, &bad_path)
-                           : row_ptr<DT>(drafter, r - BP, V);
-  const int64_t v0 = int64_t(j) * chunk_of<DT>();
   float x[kS];
   if (VEC && DT != HS_FP32) {  // all 16 loads in flight first, then the widening
     uint4 raw[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
       const int64_t v = v0 + int64_t(u * kThreads + threadIdx.x) * kV;
-      raw[u] = v < V ? __ldg(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(row) + v))
-                     : make_uint4(DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
-                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
-                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
-                                  DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u);
+      raw[u] = FULL || v < V
+                   ? __ldg(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(row) + v))
+                   : make_uint4(DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u,
+                                DT == HS_BF16 ? 0xFF80FF80u : 0xFC00FC00u);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
@@ -79,17 +73,42 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
     load_chunk<DT, VEC, kThreads, kUnroll>(row, v0, V, x);
   }
   // slots visit increasing v, so a strict '>' keeps the first index; a NaN
-  // replaces m and then stays
-  float m = -INFINITY;
-  int arg = INT_MAX;
+  // replaces m and then stays.  The winning slot is kept as its (constant)
+  // number and turned into an index once.
+  m = -INFINITY;
+  int best = -1;
 #pragma unroll
   for (int s = 0; s < kS; ++s) {
-    const int64_t v = slot_pos<DT, VEC, kThreads>(v0, s, threadIdx.x);
-    if (v < V && (x[s] > m || x[s] != x[s])) {
+    if ((FULL || slot_pos<DT, VEC, kThreads>(v0, s, threadIdx.x) < V) &&
+        (x[s] > m || x[s] != x[s])) {
       m = x[s];
-      arg = int(v);
+      best = s;
     }
   }
+  arg = best < 0 ? INT_MAX : int(slot_pos<DT, VEC, kThreads>(v0, best, threadIdx.x));
+}
+
+template <int DT, bool VEC>
+__global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
+    const void* __restrict__ target, const int32_t* __restrict__ path, int M,
+    const void* __restrict__ drafter, int B, int P, int V, Part* __restrict__ parts,
+    int nchunk) {
+  pdl_wait();
+  __shared__ float red_m[kWarps];
+  __shared__ int red_a[kWarps];
+  const int64_t r = blockIdx.x;
+  const int j = blockIdx.y;
+  const int64_t BP = int64_t(B) * P;
+  bool bad_path = false;
+  const void* row = r < BP ? target_row<DT>(target, path, M, P, r, V, &bad_path)
+                           : row_ptr<DT>(drafter, r - BP, V);
+  const int64_t v0 = int64_t(j) * chunk_of<DT>();
+  float m;
+  int arg;
+  if (v0 + chunk_of<DT>() <= V)  // every chunk but a ragged last one
+    chunk_argmax<DT, VEC, true>(row, v0, V, m, arg);
+  else
+    chunk_argmax<DT, VEC, false>(row, v0, V, m, arg);
   const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
   const float wm = warp_max_nan(m);
   const int wa = warp_min_int(m == wm ? arg : INT_MAX);
