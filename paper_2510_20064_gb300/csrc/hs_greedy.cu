@@ -5,8 +5,8 @@
 //                           max of the stored logits and the first index
 //                           holding it; every logit is read once, each thread
 //                           issuing its 16 16-byte loads before using any;
-//                           only a row's ragged last chunk checks each slot
-//                           against V
+//                           slots past the row's end hold -inf, which never
+//                           wins, so no slot is checked against V
 //   greedy_finalize_kernel  one warp per (drafter i, query b), lane k for
 //                           position k: combines the chunk partials of its
 //                           target and drafter rows in chunk order (first
@@ -36,7 +36,7 @@ __host__ __device__ constexpr int64_t chunk_of() {
 
 // This thread's max of one chunk of a row and the first index holding it
 // (INT_MAX when the chunk has no logit above -inf).  FULL: the chunk lies
-// inside the row, so no slot needs a bounds check.
+// inside the row, so no load needs a bounds check.
 template <int DT, bool VEC, bool FULL>
 __device__ __forceinline__ void chunk_argmax(const void* row, int64_t v0, int V, float& m,
                                              int& arg) {
@@ -73,14 +73,14 @@ __device__ __forceinline__ void chunk_argmax(const void* row, int64_t v0, int V,
     load_chunk<DT, VEC, kThreads, kUnroll>(row, v0, V, x);
   }
   // slots visit increasing v, so a strict '>' keeps the first index; a NaN
-  // replaces m and then stays.  The winning slot is kept as its (constant)
-  // number and turned into an index once.
+  // replaces m and then stays; the -inf past the row's end never replaces
+  // it.  The winning slot is kept as its (constant) number and turned into
+  // an index once.
   m = -INFINITY;
   int best = -1;
 #pragma unroll
   for (int s = 0; s < kS; ++s) {
-    if ((FULL || slot_pos<DT, VEC, kThreads>(v0, s, threadIdx.x) < V) &&
-        (x[s] > m || x[s] != x[s])) {
+    if (x[s] > m || x[s] != x[s]) {
       m = x[s];
       best = s;
     }
@@ -105,7 +105,7 @@ __global__ void __launch_bounds__(kThreads) argmax_chunk_kernel(
   const int64_t v0 = int64_t(j) * chunk_of<DT>();
   float m;
   int arg;
-  if (v0 + chunk_of<DT>() <= V)  // every chunk but a ragged last one
+  if (v0 + chunk_of<DT>() <= V)  // every chunk but a ragged last one: no load predicates
     chunk_argmax<DT, VEC, true>(row, v0, V, m, arg);
   else
     chunk_argmax<DT, VEC, false>(row, v0, V, m, arg);
