@@ -363,6 +363,26 @@ __device__ __forceinline__ void topl_step(const uint4 (&cur)[kUnroll], const uin
 }
 
 // ---- segment A: a share of the target row -----------------------------------
+// Packed fp32 pairs (two lanes of one 64-bit register pair): the same IEEE
+// roundings as the scalar operations, two logits per instruction.
+__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
+  uint64_t d;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
+  return d;
+}
+__device__ __forceinline__ float lo2(uint64_t d) { return __uint_as_float(uint32_t(d)); }
+__device__ __forceinline__ float hi2(uint64_t d) { return __uint_as_float(uint32_t(d >> 32)); }
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // Per lane: running max tm (stored logit), first index of it, and the sum of
 // 2^{(z - tm) c} over the lane's logits so far (rescaled when tm grows).
 template <int DT>
@@ -383,10 +403,24 @@ __device__ __forceinline__ void stats_step(const uint4 (&cur)[kUnroll], float lm
           targ = base + (u * 32 + l) * kN + q;
   }
   if (!greedy && tm != -INFINITY) {
+    // two logits at a time: (z - tm) then times c, then 2^x (-inf -> 0),
+    // summed in two independent chains
+    const uint64_t ntm2 = pack2(-tm, -tm), c2 = pack2(c, c);
+    uint64_t sa = 0ull, sb = 0ull;
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u)
 #pragma unroll
-      for (int q = 0; q < kN; ++q) ts += ex2((Vec<DT>::at(cur[u], q) - tm) * c);  // -inf -> 0
+      for (int q = 0; q < kN; q += 2) {
+        const uint64_t z2 = pack2(Vec<DT>::at(cur[u], q), Vec<DT>::at(cur[u], q + 1));
+        const uint64_t e = mul2(add2(z2, ntm2), c2);
+        const uint64_t x = pack2(ex2(lo2(e)), ex2(hi2(e)));
+        if ((q >> 1) & 1)
+          sb = add2(sb, x);
+        else
+          sa = add2(sa, x);
+      }
+    const uint64_t s2 = add2(sa, sb);
+    ts += lo2(s2) + hi2(s2);
   }
 }
 
